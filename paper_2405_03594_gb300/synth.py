@@ -1,0 +1,125 @@
+"""Seeded synthetic inputs shaped like the Llama-2-7B linear layers.
+
+This module is the one piece shared by the CUDA path's tests/bench and by the
+CPU oracle's tests: it makes weights, masks, INT8 (q, s) pairs and activations,
+and holds none of the sparse-linear arithmetic itself (no compression, no
+products).  Everything is NumPy on the host, driven by
+``numpy.random.default_rng(SeedSequence([seed, layer, proj, stream]))``.
+
+Stand-ins for what the paper takes from elsewhere (Sec. 2.1, 3.4):
+  * SparseGPT masks -> per-row magnitude masks: in each row the n_prune entries
+    with the smallest |w| are dropped, ties broken by the lower column first
+    (a stable sort on |w|); n_prune = round-half-even(pct * K / 100).
+  * Outlier-aware non-uniform masks -> per-row sparsity drawn uniformly within
+    +-10 points of the target (clipped to [0, 90]), with 5% of the columns
+    (round(0.05 K), drawn once per matrix) never pruned.
+  * GPTQ/SmoothQuant INT8 -> symmetric absmax per output row over the kept
+    weights: s = max|w| / 127 (s = 1 for an empty or all-zero row),
+    q = clamp(round-half-even(w / s), -127, 127) at kept positions, 0 elsewhere.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# The four fused Llama-2-7B linear shapes (N = out features, K = in features).
+LLAMA2_7B_SHAPES = {
+    "qkv": (12288, 4096),
+    "o": (4096, 4096),
+    "gate_up": (22016, 4096),
+    "down": (4096, 11008),
+}
+PROJ_IDS = {"qkv": 0, "o": 1, "gate_up": 2, "down": 3, "q": 4}
+STREAM_W, STREAM_MASK, STREAM_X, STREAM_RESID = 0, 1, 2, 3
+
+
+def rng(seed: int, layer: int, proj: int, stream: int) -> np.random.Generator:
+    return np.random.default_rng(np.random.SeedSequence([seed, layer, proj, stream]))
+
+
+def bf16_from_f32(a: np.ndarray) -> np.ndarray:
+    """float32 -> bf16 bit patterns (uint16), round to nearest even.  Finite inputs."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    r = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return r.astype(np.uint16)
+
+
+def bf16_to_f32(h: np.ndarray) -> np.ndarray:
+    return (np.ascontiguousarray(h, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def round_half_even_div(num: int, den: int) -> int:
+    q, r = divmod(num, den)
+    if 2 * r > den or (2 * r == den and q % 2 == 1):
+        q += 1
+    return q
+
+
+def n_pruned(pct: int, K: int) -> int:
+    """Entries dropped per row at an integer sparsity percentage."""
+    return round_half_even_div(pct * K, 100)
+
+
+def weight(N: int, K: int, g: np.random.Generator, std: float = 0.02) -> np.ndarray:
+    """bf16 bits of W ~ N(0, std^2), shape [N, K]."""
+    return bf16_from_f32(g.standard_normal((N, K), dtype=np.float32) * np.float32(std))
+
+
+def activations(M: int, K: int, g: np.random.Generator) -> np.ndarray:
+    """bf16 bits of x ~ N(0, 1), shape [M, K]."""
+    return bf16_from_f32(g.standard_normal((M, K), dtype=np.float32))
+
+
+def _prune_smallest(absw: np.ndarray, n_prune_per_row: np.ndarray, keep_cols=None) -> np.ndarray:
+    N, K = absw.shape
+    a = absw.copy()
+    if keep_cols is not None:
+        a[:, keep_cols] = np.inf  # never chosen before any prunable column
+    order = np.argsort(a, axis=1, kind="stable")
+    rank = np.empty_like(order)
+    rows = np.arange(N)[:, None]
+    rank[rows, order] = np.arange(K)[None, :]
+    return (rank >= n_prune_per_row[:, None]).astype(np.uint8)
+
+
+def magnitude_mask(W: np.ndarray, pct: int) -> np.ndarray:
+    """uint8 keep-mask [N, K]: per row, drop the n_pruned(pct, K) smallest |w|."""
+    N, K = W.shape
+    absw = np.abs(bf16_to_f32(W))
+    n = np.full(N, n_pruned(pct, K), dtype=np.int64)
+    return _prune_smallest(absw, n)
+
+
+def nonuniform_mask(W: np.ndarray, pct: int, g: np.random.Generator):
+    """Non-uniform per-row magnitude mask with dense outlier columns.
+
+    Returns (mask, n_prune_per_row, outlier_cols)."""
+    N, K = W.shape
+    n_out = round_half_even_div(5 * K, 100)
+    outliers = np.sort(g.choice(K, size=n_out, replace=False))
+    s_row = np.clip(g.uniform(pct - 10.0, pct + 10.0, size=N), 0.0, 90.0)
+    n_prune = np.rint(s_row * K / 100.0).astype(np.int64)
+    n_prune = np.minimum(np.maximum(n_prune, 0), K - n_out)
+    if pct == 0:
+        n_prune[:] = 0
+    absw = np.abs(bf16_to_f32(W))
+    return _prune_smallest(absw, n_prune, outliers), n_prune, outliers
+
+
+def quantize_int8(W: np.ndarray, mask: np.ndarray):
+    """(q int8 [N, K], s float32 [N]) by symmetric absmax over the kept weights."""
+    w = bf16_to_f32(W).astype(np.float64) * (mask != 0)
+    amax = np.abs(w).max(axis=1)
+    s = np.where(amax > 0, amax / 127.0, 1.0).astype(np.float32)
+    q = np.clip(np.rint(w / s.astype(np.float64)[:, None]), -127, 127).astype(np.int8)
+    q[mask == 0] = 0
+    return q, s
+
+
+def layer_inputs(shape_name: str, pct: int, M: int, seed: int = 0, layer: int = 0):
+    """(W, mask, x) for one Llama-2-7B linear at a uniform per-row sparsity."""
+    N, K = LLAMA2_7B_SHAPES[shape_name]
+    p = PROJ_IDS[shape_name]
+    W = weight(N, K, rng(seed, layer, p, STREAM_W))
+    mask = magnitude_mask(W, pct)
+    x = activations(M, K, rng(seed, layer, p, STREAM_X))
+    return W, mask, x

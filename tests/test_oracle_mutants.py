@@ -1,0 +1,75 @@
+"""The oracle's pins must be sharp: plant one plausible mistake at a time in a copy of
+sp_oracle.c (on the CPU), rebuild it, and check that at least one pin fails."""
+import os
+import subprocess
+
+import pytest
+
+import oracle as oracle_mod
+from tests import test_oracle as pins
+
+SRC = os.path.join(os.path.dirname(oracle_mod.__file__), "sp_oracle.c")
+
+MUTANTS = {
+    "sum_sign": ("acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);",
+                 "acc -= or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);"),
+    "transposed_x": ("acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);",
+                     "acc += or_bf16_to_double(x[k * M + m]) * or_bf16_to_double(W[n * K + k]);"),
+    "dropped_first_term": ("for (int64_t k = 0; k < K; ++k)\n        if (mask[n * K + k]) acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W",
+                           "for (int64_t k = 1; k < K; ++k)\n        if (mask[n * K + k]) acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W"),
+    "mask_msb_first": ("if (k < K && mask[n * K + k]) m |= (uint64_t)1 << j;",
+                       "if (k < K && mask[n * K + k]) m |= (uint64_t)1 << (63 - j);"),
+    "pad_to_8": ("#define OR_ALIGN 16", "#define OR_ALIGN 8"),
+    "int8_scale_dropped": ("acc += or_bf16_to_double(x[m * K + k]) * ((double)q[n * K + k] * sn);",
+                           "acc += or_bf16_to_double(x[m * K + k]) * ((double)q[n * K + k]);"),
+    "block_mask_msb_first": ("m |= (uint64_t)1 << i;", "m |= (uint64_t)1 << (n - 1 - i);"),
+    "bf16_shift": ("uint32_t u = (uint32_t)h << 16;", "uint32_t u = (uint32_t)h << 15;"),
+    "tile_width_off_by_one": ("for (int j = 0; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals",
+                              "for (int j = 1; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals"),
+}
+
+
+def _pin_suite(o):
+    """Run a fixed selection of pins against whatever library `o` is bound to; return
+    the names of those that failed."""
+    checks = {
+        "paper_example": lambda: pins.test_paper_example_register_layout_and_encoding(o),
+        "format_bytes": lambda: pins.test_format_hand_derived_bytes(o),
+        "format_linear": lambda: pins.test_format_hand_derived_linear(o),
+        "roundtrip": lambda: pins.test_roundtrip_bit_exact(o, 300, 200, 70, False),
+        "roundtrip_int8": lambda: pins.test_roundtrip_bit_exact(o, 130, 72, 50, True),
+        "layout": lambda: pins.test_layout_invariants(o, 257, 136),
+        "integer_exact": lambda: pins.test_linear_integer_valued_exact(o, 40, 136, 3),
+        "library_matmul": lambda: pins.test_linear_matches_float64_library_matmul(o, 70),
+        "one_hot": lambda: pins.test_linear_one_hot_selects_a_column(o),
+        "int8_exact": lambda: pins.test_int8_oracle_integer_exact_and_scale(o),
+    }
+    failed = []
+    for name, fn in checks.items():
+        try:
+            fn()
+        except (AssertionError, ValueError):
+            failed.append(name)
+    return failed
+
+
+def test_unmutated_oracle_passes_the_suite(oracle):
+    assert _pin_suite(oracle) == []
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_each_planted_mistake_is_caught(oracle, tmp_path, name):
+    old, new = MUTANTS[name]
+    src = open(SRC).read()
+    assert src.count(old) >= 1, f"mutation anchor for {name} not found"
+    mutated = src.replace(old, new, 1)
+    path_c = tmp_path / "mut.c"
+    path_c.write_text(mutated)
+    so = tmp_path / "libmut.so"
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", str(path_c), "-o", str(so)])
+    oracle_mod.use_library(str(so))
+    try:
+        failed = _pin_suite(oracle_mod)
+    finally:
+        oracle_mod.use_library(None)
+    assert failed, f"mutant {name} survived every pin"
