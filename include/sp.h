@@ -1,0 +1,154 @@
+/*
+ * sp.h -- C ABI of libsp: bitmask-compressed unstructured-sparse linear layers
+ * y = x . (W o Mask)^T on one NVIDIA GB300 (sm_103a).
+ *
+ * Method.  The weight is stored the way the paper's GPU engine stores it
+ * (Sec. 2.4.2): cut into submatrices, each kept as its dense nonzero values plus
+ * a bitmask; at run time the submatrices are streamed from global memory and
+ * expanded on chip by the bitmask (the per-block bitmask encoding itself is the
+ * one of Sec. 2.4.1).  Decode-sized batches are bound by reading the compressed
+ * bytes; prefill-sized batches run the expanded tiles on the tensor cores.
+ *
+ * Compressed format (identical bytes on every GPU; see also the constants below).
+ *   The matrix [N, K] is cut into T = ceil(K/64) K-tiles and RB = ceil(N/128)
+ *   row blocks.  Chunk (rb, t) is number c = rb*T + t and starts at byte off[c]
+ *   of the buffer (off[0] = 0, off[RB*T] = total size, all multiples of 16):
+ *     bytes [0, 1024)   128 little-endian uint64 masks, one per row 128*rb + r;
+ *                       bit j (LSB = 0) set <=> column 64*t + j is kept.
+ *                       Rows >= N and columns >= K have no bits.
+ *     then              the kept values of row 0, row 1, ..., row 127 of the
+ *                       chunk, each row in ascending column order (bf16 bit
+ *                       patterns, 2 bytes; or int8, 1 byte), no gaps;
+ *     then              zero bytes up to the next multiple of 16.
+ *   INT8 matrices also carry one fp32 scale per output row: w[n,k] = q[n,k]*s[n].
+ *
+ * Conventions for every call.
+ *   - Device pointers point to memory of the current CUDA device, row-major and
+ *     contiguous, and must be 16-byte aligned (else SP_ERR_ALIGNMENT).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  Calls are asynchronous on that stream unless stated otherwise;
+ *     the caller keeps every buffer alive until the stream has passed the call.
+ *   - No call aborts, traps or prints.  Every call returns a status.  Kernel
+ *     waits are bounded: a wait that expires records SP_ERR_TIMEOUT in a device
+ *     status word that sp_check() reports.
+ *   - There is no CPU fallback: without a usable GPU the calls that need one
+ *     return SP_ERR_CUDA.
+ */
+#ifndef SP_H
+#define SP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SP_TILE_K 64            /* columns per K-tile (one uint64 mask per row) */
+#define SP_CHUNK_ROWS 128       /* rows per chunk */
+#define SP_CHUNK_MASK_BYTES 1024
+#define SP_CHUNK_ALIGN 16
+
+typedef enum sp_status {
+  SP_OK = 0,
+  SP_ERR_INVALID_ARG = 1,   /* null pointer, negative or zero size, bad enum */
+  SP_ERR_UNSUPPORTED = 2,   /* valid but not supported (e.g. K % 8 != 0) */
+  SP_ERR_ALIGNMENT = 3,     /* a pointer is not 16-byte aligned */
+  SP_ERR_CUDA = 4,          /* a CUDA runtime call or a launch failed */
+  SP_ERR_OUT_OF_MEMORY = 5, /* the allocator returned NULL */
+  SP_ERR_TIMEOUT = 6,       /* a bounded device wait expired (reported by sp_check) */
+  SP_ERR_BAD_HANDLE = 7,    /* not a live sp_matrix */
+  SP_ERR_WORKSPACE = 8      /* workspace missing or smaller than sp_workspace_size() */
+} sp_status;
+
+typedef enum sp_dtype { SP_BF16 = 0, SP_INT8 = 1 } sp_dtype;
+
+/* Kernel family used by sp_linear_ex.  SP_PATH_AUTO picks by batch size M. */
+typedef enum sp_path {
+  SP_PATH_AUTO = 0,
+  SP_PATH_CUDA_CORE = 1,    /* popc-prefix expansion, FP32 FMA on CUDA cores */
+  SP_PATH_TENSOR_CORE = 2   /* expansion into tensor memory, tcgen05 MMA */
+} sp_path;
+
+typedef struct sp_matrix sp_matrix; /* opaque; owns the compressed weight */
+
+typedef struct sp_info_t {
+  int64_t n, k;             /* logical shape [N, K] */
+  int64_t tiles, row_blocks;
+  int32_t dtype;            /* sp_dtype */
+  int32_t device;           /* CUDA device the buffers live on */
+  int64_t nnz;              /* kept entries */
+  uint64_t bytes;           /* size of the compressed buffer (padding included) */
+  uint64_t max_chunk_bytes; /* largest single chunk */
+  uint64_t scale_bytes;     /* 4*N for INT8, else 0 */
+} sp_info_t;
+
+/* Device allocator callbacks.  alloc returns a device pointer of at least `bytes`
+ * bytes, 256-byte aligned, or NULL; free releases it.  Passing NULL for both uses
+ * cudaMalloc / cudaFree.  The library calls them only inside sp_compress,
+ * sp_clone and sp_free. */
+typedef void* (*sp_alloc_fn)(size_t bytes, void* ctx);
+typedef void (*sp_free_fn)(void* ptr, void* ctx);
+
+/* Compress W o Mask (the storage of Sec. 2.4.2).
+ *   w_dev      [N, K] bf16 bit patterns (SP_BF16) or int8 values (SP_INT8).
+ *   mask_dev   [N, K] uint8, nonzero = kept.  A kept zero is stored as a value;
+ *              a masked-out nonzero is dropped.
+ *   scale_dev  [N] fp32 per-row scales for SP_INT8 (copied); must be NULL for SP_BF16.
+ *   N, K       N >= 1, K >= 1, K % 8 == 0 (SP_ERR_UNSUPPORTED otherwise).
+ * Synchronises `stream` once (the total size sizes the buffer).  On success *out
+ * is a new handle owning its device buffers; on error *out is NULL and nothing
+ * is leaked.  Inputs are only read and may be freed once the call returns. */
+sp_status sp_compress(const void* w_dev, const uint8_t* mask_dev, int64_t n, int64_t k, sp_dtype dtype,
+                      const float* scale_dev, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx,
+                      void* stream, sp_matrix** out);
+
+/* Expand the handle back to the dense masked weight: w_out_dev [N, K] of the
+ * handle's dtype, zero where masked out, bit-exact. */
+sp_status sp_decompress(const sp_matrix* h, void* w_out_dev, void* stream);
+
+/* Bytes of device workspace that sp_linear needs for a batch of m rows (may be 0). */
+sp_status sp_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
+
+/* y = x . (W o Mask)^T, FP32 accumulation, bf16 output (round to nearest even).
+ *   x_dev      [m, K] bf16.      y_dev [m, N] bf16 (fully overwritten).
+ *   workspace  device memory of at least sp_workspace_size(h, m) bytes, zero-filled
+ *              before its first use; every call leaves it ready for the next one.
+ *              Calls that share a workspace must be ordered on one stream.
+ *   m == 0 returns SP_OK without a launch.  No allocation, no host sync: the call
+ *   can be captured in a CUDA graph.  Results are bitwise repeatable for a given
+ *   (matrix, m, device). */
+sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
+                    size_t workspace_bytes, void* stream);
+
+/* sp_linear with an explicit kernel family (tests run each family on its own). */
+sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
+                       size_t workspace_bytes, sp_path path, void* stream);
+
+/* A copy of the handle with its own device buffers (same bytes). */
+sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx, void* stream,
+                   sp_matrix** out);
+
+/* Release the handle and its device buffers.  The caller must ensure no queued
+ * work still reads them (e.g. synchronise the stream first).  NULL is a no-op. */
+sp_status sp_free(sp_matrix* h);
+
+sp_status sp_info(const sp_matrix* h, sp_info_t* info);
+
+/* Synchronously copy the compressed bytes (info.bytes) and the RB*T+1 chunk
+ * offsets (uint64) to host memory; either destination may be NULL. */
+sp_status sp_copy_out(const sp_matrix* h, void* buf_host, size_t buf_cap, uint64_t* off_host, size_t off_count);
+
+/* Synchronise `stream`; report and clear the current device's status word.
+ * Returns SP_ERR_TIMEOUT if a kernel's bounded wait expired since the last
+ * check, SP_ERR_CUDA if the stream reported an error, else SP_OK. */
+sp_status sp_check(void* stream);
+
+/* Static English name of a status code. */
+const char* sp_status_string(sp_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SP_H */

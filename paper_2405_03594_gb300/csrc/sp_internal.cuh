@@ -1,0 +1,169 @@
+// sp_internal.cuh -- internals shared by the libsp translation units: the handle,
+// kernel parameter blocks, and thin inline-PTX wrappers for sm_103a (mbarrier,
+// bulk copies, named barriers, global timer).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/sp.h"
+
+#define SP_MAGIC 0x53504d31u  // "SPM1"
+
+struct sp_matrix {
+  uint32_t magic;
+  int64_t N, K;
+  int32_t T, RB;
+  sp_dtype dtype;
+  int32_t esize;
+  int64_t nnz;
+  uint64_t bytes;
+  uint64_t max_chunk;
+  uint8_t* d_buf;
+  uint64_t* d_off;
+  float* d_scale;
+  sp_alloc_fn alloc;
+  sp_free_fn free_fn;
+  void* ctx;
+  int32_t device;
+  int32_t num_sms;
+};
+
+namespace sp {
+
+constexpr int kTileK = SP_TILE_K;
+constexpr int kRows = SP_CHUNK_ROWS;
+constexpr int kMaskBytes = SP_CHUNK_MASK_BYTES;
+
+// Work decomposition shared by every sp_linear kernel ("stream-K" over chunks).
+// The W = MT * RB * T work items (token tile mt, chunk c = rb*T + t) are cut into G
+// contiguous ranges, CTA i taking [i*W/G, (i+1)*W/G).  A (mt, rb) pair whose T
+// chunks all fall in one CTA is finished there; otherwise every contributing CTA
+// stores a fp32 partial in its slot (0 = its first segment, 1 = its last), and the
+// last one to arrive sums the partials in CTA order and writes y.
+__host__ __device__ inline int64_t imin64(int64_t a, int64_t b) { return a < b ? a : b; }
+__host__ __device__ inline int64_t range_begin(int64_t i, int64_t W, int64_t G) { return i * W / G; }
+__host__ __device__ inline int64_t owner_of(int64_t w, int64_t W, int64_t G) { return ((w + 1) * G - 1) / W; }
+
+struct LinearParams {
+  const uint8_t* buf;
+  const uint64_t* off;
+  const float* scale;   // INT8 only
+  const uint16_t* x;    // bf16 bits [M, K]
+  uint16_t* y;          // bf16 bits [M, N]
+  float* ws;            // partials [2G][kRows][Mt]
+  int* cnt;             // arrival counters [2G]
+  int* status;
+  int64_t N, K;
+  int32_t T, RB;
+  int32_t M;            // rows of x handled by this launch
+  int64_t W;            // work items
+  int32_t G;            // CTAs
+  int32_t slots;        // ring slots
+  uint32_t slot_bytes;  // bytes per ring slot (chunk region + x tile region)
+  uint32_t chunk_region;// bytes reserved for the chunk inside a slot
+  uint64_t timeout_ns;
+};
+
+// Workspace layout, fixed per device so that calls with different grids can share it:
+// [arrival counters for up to 2 * kMaxGridPerSm * SMs partial slots][fp32 partials].
+// Every call leaves the counters at zero.
+constexpr int kMaxGridPerSm = 4;
+inline size_t ws_counter_bytes(int num_sms) {
+  return ((size_t)2 * kMaxGridPerSm * num_sms * sizeof(int) + 255) / 256 * 256;
+}
+
+enum : int { kStatusOk = 0, kStatusTimeout = 1, kStatusBadFormat = 2 };
+
+// ---------------------------------------------------------------- device helpers
+#if defined(__CUDACC__)
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity.  Returns false once
+// `timeout_ns` of global time has passed without completion.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (true) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > timeout_ns) return false;
+  }
+}
+// 1-D bulk copy global -> shared, completing `bytes` of transaction on `bar`.
+// dst, src and bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_g2s_hint(void* dst, const void* src, uint32_t bytes, uint64_t* bar,
+                                              uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+__device__ __forceinline__ void set_status(int* status, int code) {
+  if (status) atomicCAS(status, kStatusOk, code);
+}
+__device__ __forceinline__ float bf16_bits_to_float(uint32_t h) { return __uint_as_float(h << 16); }
+__device__ __forceinline__ uint16_t float_to_bf16_bits_rn(float f) {
+  return __bfloat16_as_ushort(__float2bfloat16_rn(f));
+}
+#endif
+
+// ---------------------------------------------------------------- host-side entry points between TUs
+sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t K, sp_dtype dt, const float* scale,
+                          sp_alloc_fn alloc, sp_free_fn free_fn, void* ctx, cudaStream_t stream, sp_matrix** out);
+sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream);
+sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
+                           cudaStream_t stream);
+size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
+int* device_status_ptr();            // this device's status word (device address)
+uint64_t wait_timeout_ns();          // bounded-wait limit for kernels
+void* dev_alloc(const sp_matrix* h, size_t bytes);
+void dev_free(const sp_matrix* h, void* p);
+
+}  // namespace sp

@@ -1,0 +1,216 @@
+"""Thin ctypes binding of libsp (include/sp.h).  Argument marshalling only: every
+step of compression and of the sparse product runs in the library's CUDA kernels.
+PyTorch supplies device memory (through the allocator callbacks) and streams.
+
+Importing this module loads libsp.so and raises if it is missing: there is no CPU
+or PyTorch fallback for any operation here.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libsp.so")
+
+SP_BF16, SP_INT8 = 0, 1
+PATHS = {"auto": 0, "cuda_core": 1, "tensor_core": 2}
+STATUS = {
+    0: "SP_OK", 1: "SP_ERR_INVALID_ARG", 2: "SP_ERR_UNSUPPORTED", 3: "SP_ERR_ALIGNMENT", 4: "SP_ERR_CUDA",
+    5: "SP_ERR_OUT_OF_MEMORY", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_BAD_HANDLE", 8: "SP_ERR_WORKSPACE",
+}
+# every function declared in include/sp.h
+EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_clone", "sp_free",
+           "sp_info", "sp_copy_out", "sp_check", "sp_status_string"]
+
+
+class SpError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {STATUS.get(code, code)}")
+
+
+class SpInfo(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("k", ctypes.c_int64), ("tiles", ctypes.c_int64),
+                ("row_blocks", ctypes.c_int64), ("dtype", ctypes.c_int32), ("device", ctypes.c_int32),
+                ("nnz", ctypes.c_int64), ("bytes", ctypes.c_uint64), ("max_chunk_bytes", ctypes.c_uint64),
+                ("scale_bytes", ctypes.c_uint64)]
+
+
+ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
+FREE_FN = ctypes.CFUNCTYPE(None, ctypes.c_void_p, ctypes.c_void_p)
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    if not os.path.exists(path):
+        raise ImportError(f"libsp.so not built at {path}: run __graft_entry__.build() (no fallback exists)")
+    lib = ctypes.CDLL(path)
+    P, I64, SZ = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t
+    lib.sp_compress.argtypes = [P, P, I64, I64, ctypes.c_int, P, ALLOC_FN, FREE_FN, P, P, ctypes.POINTER(P)]
+    lib.sp_decompress.argtypes = [P, P, P]
+    lib.sp_workspace_size.argtypes = [P, I64, ctypes.POINTER(SZ)]
+    lib.sp_linear.argtypes = [P, P, I64, P, P, SZ, P]
+    lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
+    lib.sp_clone.argtypes = [P, ALLOC_FN, FREE_FN, P, P, ctypes.POINTER(P)]
+    lib.sp_free.argtypes = [P]
+    lib.sp_info.argtypes = [P, ctypes.POINTER(SpInfo)]
+    lib.sp_copy_out.argtypes = [P, P, SZ, P, SZ]
+    lib.sp_check.argtypes = [P]
+    lib.sp_status_string.argtypes = [ctypes.c_int]
+    lib.sp_status_string.restype = ctypes.c_char_p
+    for name in EXPORTS:
+        if name != "sp_status_string":
+            getattr(lib, name).restype = ctypes.c_int
+    return lib
+
+
+_lib = load_library()
+
+# ------------------------------------------------------------------ torch-backed allocator
+_live = {}
+_live_lock = threading.Lock()
+
+
+def _alloc(nbytes, ctx):
+    try:
+        t = torch.empty(int(nbytes), dtype=torch.uint8, device=torch.device("cuda", torch.cuda.current_device()))
+    except Exception:
+        return None
+    p = t.data_ptr()
+    with _live_lock:
+        _live[p] = t
+    return p
+
+
+def _free(ptr, ctx):
+    with _live_lock:
+        _live.pop(ptr, None)
+
+
+_ALLOC = ALLOC_FN(_alloc)
+_FREE = FREE_FN(_free)
+
+
+def _check(code: int, where: str):
+    if code != 0:
+        raise SpError(code, where)
+
+
+def _stream(stream=None) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t: torch.Tensor | None) -> ctypes.c_void_p:
+    return ctypes.c_void_p(0 if t is None else t.data_ptr())
+
+
+class SparseMatrix:
+    """A compressed weight owned by libsp (the handle) with torch-allocated buffers."""
+
+    def __init__(self, handle: ctypes.c_void_p):
+        self._h = handle
+        info = SpInfo()
+        _check(_lib.sp_info(self._h, ctypes.byref(info)), "sp_info")
+        self.info = info
+        self.n, self.k = int(info.n), int(info.k)
+        self.dtype = "int8" if info.dtype == SP_INT8 else "bf16"
+
+    @property
+    def handle(self):
+        return self._h
+
+    def workspace_size(self, m: int) -> int:
+        b = ctypes.c_size_t()
+        _check(_lib.sp_workspace_size(self._h, m, ctypes.byref(b)), "sp_workspace_size")
+        return int(b.value)
+
+    def linear(self, x: torch.Tensor, out: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
+               path: str = "auto", stream=None) -> torch.Tensor:
+        """y = x . (W o Mask)^T with x [m, K] bf16 on this matrix's device."""
+        assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
+        m = x.shape[0]
+        if out is None:
+            out = torch.empty((m, self.n), dtype=torch.bfloat16, device=x.device)
+        if workspace is None:
+            workspace = workspace_for(self.workspace_size(m), x.device)
+        _check(_lib.sp_linear_ex(self._h, _ptr(x), m, _ptr(out), _ptr(workspace), workspace.numel(), PATHS[path],
+                                 _stream(stream)), "sp_linear")
+        return out
+
+    def decompress(self, stream=None) -> torch.Tensor:
+        dt = torch.int8 if self.dtype == "int8" else torch.bfloat16
+        out = torch.empty((self.n, self.k), dtype=dt, device=torch.device("cuda", int(self.info.device)))
+        _check(_lib.sp_decompress(self._h, _ptr(out), _stream(stream)), "sp_decompress")
+        return out
+
+    def copy_out(self) -> tuple[np.ndarray, np.ndarray]:
+        buf = np.zeros(max(int(self.info.bytes), 1), dtype=np.uint8)
+        off = np.zeros(int(self.info.tiles * self.info.row_blocks + 1), dtype=np.uint64)
+        _check(_lib.sp_copy_out(self._h, buf.ctypes.data_as(ctypes.c_void_p), buf.size,
+                                off.ctypes.data_as(ctypes.c_void_p), off.size), "sp_copy_out")
+        return buf[:int(self.info.bytes)], off
+
+    def clone(self, stream=None) -> "SparseMatrix":
+        h = ctypes.c_void_p()
+        _check(_lib.sp_clone(self._h, _ALLOC, _FREE, None, _stream(stream), ctypes.byref(h)), "sp_clone")
+        return SparseMatrix(h)
+
+    def free(self):
+        if self._h:
+            torch.cuda.synchronize()
+            _check(_lib.sp_free(self._h), "sp_free")
+            self._h = None
+
+    def __del__(self):
+        try:
+            if self._h:
+                _lib.sp_free(self._h)
+                self._h = None
+        except Exception:
+            pass
+
+
+def compress(w: torch.Tensor, mask: torch.Tensor, scale: torch.Tensor | None = None, stream=None) -> SparseMatrix:
+    """Compress W o mask.  w: [N, K] bf16 (or int8 with scale [N] fp32); mask: [N, K] uint8/bool."""
+    assert w.is_cuda and w.dim() == 2 and w.is_contiguous()
+    if mask.dtype == torch.bool:
+        mask = mask.to(torch.uint8)
+    assert mask.dtype == torch.uint8 and mask.shape == w.shape and mask.is_contiguous()
+    if w.dtype == torch.int8:
+        assert scale is not None and scale.dtype == torch.float32 and scale.numel() == w.shape[0]
+        dt = SP_INT8
+    else:
+        assert w.dtype in (torch.bfloat16, torch.int16, torch.uint16) and scale is None
+        dt = SP_BF16
+    h = ctypes.c_void_p()
+    _check(_lib.sp_compress(_ptr(w), _ptr(mask), w.shape[0], w.shape[1], dt, _ptr(scale), _ALLOC, _FREE, None,
+                            _stream(stream), ctypes.byref(h)), "sp_compress")
+    return SparseMatrix(h)
+
+
+_ws_cache: dict = {}
+
+
+def workspace_for(nbytes: int, device) -> torch.Tensor:
+    """A zero-filled workspace of at least nbytes on `device`, shared by calls on one stream."""
+    dev = torch.device(device)
+    key = dev.index if dev.index is not None else torch.cuda.current_device()
+    ws = _ws_cache.get(key)
+    if ws is None or ws.numel() < max(nbytes, 1):
+        ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=torch.device("cuda", key))
+        _ws_cache[key] = ws
+    return ws
+
+
+def check(stream=None):
+    """Synchronise the stream and raise if a kernel's bounded wait expired."""
+    _check(_lib.sp_check(_stream(stream)), "sp_check")
+
+
+def status_string(code: int) -> str:
+    return _lib.sp_status_string(code).decode()

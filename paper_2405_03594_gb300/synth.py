@@ -37,10 +37,14 @@ def rng(seed: int, layer: int, proj: int, stream: int) -> np.random.Generator:
 
 
 def bf16_from_f32(a: np.ndarray) -> np.ndarray:
-    """float32 -> bf16 bit patterns (uint16), round to nearest even.  Finite inputs."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    r = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
-    return r.astype(np.uint16)
+    """float32 -> bf16 bit patterns (uint16), round to nearest even.  Finite inputs
+    (the largest finite pattern plus the rounding bias still fits in 32 bits)."""
+    u = np.array(a, dtype=np.float32, copy=True).view(np.uint32)
+    lsb = (u >> 16) & 1
+    u += 0x7FFF
+    u += lsb
+    u >>= 16
+    return u.astype(np.uint16)
 
 
 def bf16_to_f32(h: np.ndarray) -> np.ndarray:
@@ -69,24 +73,37 @@ def activations(M: int, K: int, g: np.random.Generator) -> np.ndarray:
     return bf16_from_f32(g.standard_normal((M, K), dtype=np.float32))
 
 
-def _prune_smallest(absw: np.ndarray, n_prune_per_row: np.ndarray, keep_cols=None) -> np.ndarray:
-    N, K = absw.shape
-    a = absw.copy()
+def _prune_smallest(W: np.ndarray, n_prune_per_row: np.ndarray, keep_cols=None) -> np.ndarray:
+    """Keep-mask dropping, per row, the n smallest |w| with ties broken by the lower
+    column.  Every entry gets the unique key (|w| bit pattern, column): for
+    non-negative floats the bit pattern orders like the value, so the n smallest
+    keys are exactly the first n entries of a stable sort on |w|."""
+    N, K = W.shape
+    assert K < (1 << 20)
+    key = (np.ascontiguousarray(W, dtype=np.uint16) & np.uint16(0x7FFF)).astype(np.uint64)
+    key <<= np.uint64(20)
+    key |= np.arange(K, dtype=np.uint64)[None, :]
     if keep_cols is not None:
-        a[:, keep_cols] = np.inf  # never chosen before any prunable column
-    order = np.argsort(a, axis=1, kind="stable")
-    rank = np.empty_like(order)
-    rows = np.arange(N)[:, None]
-    rank[rows, order] = np.arange(K)[None, :]
-    return (rank >= n_prune_per_row[:, None]).astype(np.uint8)
+        key[:, keep_cols] |= np.uint64(1) << np.uint64(40)  # after every prunable column
+    mask = np.ones((N, K), dtype=np.uint8)
+    for n in np.unique(n_prune_per_row):
+        rows = np.nonzero(n_prune_per_row == n)[0]
+        if n <= 0:
+            continue
+        if n >= K:
+            mask[rows] = 0
+            continue
+        sub = key[rows]
+        thr = np.partition(sub, n - 1, axis=1)[:, n - 1]
+        mask[rows] = (sub > thr[:, None]).astype(np.uint8)
+    return mask
 
 
 def magnitude_mask(W: np.ndarray, pct: int) -> np.ndarray:
     """uint8 keep-mask [N, K]: per row, drop the n_pruned(pct, K) smallest |w|."""
     N, K = W.shape
-    absw = np.abs(bf16_to_f32(W))
     n = np.full(N, n_pruned(pct, K), dtype=np.int64)
-    return _prune_smallest(absw, n)
+    return _prune_smallest(W, n)
 
 
 def nonuniform_mask(W: np.ndarray, pct: int, g: np.random.Generator):
@@ -101,8 +118,7 @@ def nonuniform_mask(W: np.ndarray, pct: int, g: np.random.Generator):
     n_prune = np.minimum(np.maximum(n_prune, 0), K - n_out)
     if pct == 0:
         n_prune[:] = 0
-    absw = np.abs(bf16_to_f32(W))
-    return _prune_smallest(absw, n_prune, outliers), n_prune, outliers
+    return _prune_smallest(W, n_prune, outliers), n_prune, outliers
 
 
 def quantize_int8(W: np.ndarray, mask: np.ndarray):
