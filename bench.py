@@ -1,0 +1,472 @@
+#!/usr/bin/env python
+"""Decode throughput of the Llama-2-7B sparse linear stack on GB300.
+
+A step is one decode step through the linear layers of all 32 Llama-2-7B layers:
+per layer the fused qkv (4096->12288), o (4096->4096), fused gate/up (4096->22016)
+and down (11008->4096) projections, 70% unstructured per-row magnitude sparsity,
+bf16 weights in the bitmask-compressed format, x bf16 [M, K], FP32 accumulation,
+bf16 y.  tok/s = M / step time.  The 32 layers are 32 distinct device copies of one
+seeded layer, so every step streams 4.7 GB (> L2) of compressed weights from HBM.
+
+  python bench.py [--gpus N --steps K --warmup W --m M]        our CUDA path
+  python bench.py --impl reference ...                          the float64 CPU oracle
+
+One JSON line on stdout (rank 0).  With --gpus N > 1 (under torchrun) every rank
+runs an independent replica (weak scaling; no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Llama-2-7B sparse-linear decode tok/s @70%; achieved HBM GB/s vs roofline"
+SHAPES = ["qkv", "o", "gate_up", "down"]
+LAYERS = 32
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--m", type=int, default=16, help="decode batch (tokens per step)")
+    ap.add_argument("--pct", type=int, default=70)
+    ap.add_argument("--path", default="auto", choices=["auto", "cuda_core", "tensor_core"])
+    ap.add_argument("--sweep", default="1,4,16", help="extra batch sizes reported under per_m ('' = none)")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle leg")
+    ap.add_argument("--single", default="", choices=["", *SHAPES],
+                    help="profiling aid: time one layer-0 linear of this shape (--warmup then --steps launches)")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+def host_layer(pct: int, M: int):
+    """Seeded host inputs of layer 0: W, mask and x per shape (the oracle's inputs)."""
+    from paper_2405_03594_gb300 import synth
+
+    out = {}
+    for name in SHAPES:
+        W, mask, x = synth.layer_inputs(name, pct, M, seed=0, layer=0)
+        out[name] = (W, mask, x)
+    return out
+
+
+def algorithmic_bytes(info, M: int, K: int, N: int) -> int:
+    """Compressed-weight bytes the method must read (values + one bit per weight,
+    plus INT8 scales) plus the activations read and the outputs written."""
+    esize = 1 if info.dtype == 1 else 2
+    return int(info.nnz) * esize + N * K // 8 + int(info.scale_bytes) + 2 * M * K + 2 * M * N
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2405_03594_gb300", "csrc")
+    for n in sorted(os.listdir(csrc)):
+        if n.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, n), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the
+    current kernel sources; else None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(f"{kernel}|{workload}")
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.gpu = gpu_index
+        self.p = None
+
+    def __enter__(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.p:
+            time.sleep(0.2)
+            self.p.terminate()
+            self.p.wait()
+
+    def summary(self):
+        self.f.flush()
+        self.f.seek(0)
+        rows = [r.strip().split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [c.strip() for c in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, r[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def cpu_oracle_leg(host, M: int, reps_target_s: float = 10.0):
+    """Time the float64 oracle on this host's cores on layer 0 (all four linears) and
+    scale to a 32-layer step.  Returns (cpu_baseline dict, oracle outputs)."""
+    cores = len(os.sched_getaffinity(0))
+    os.environ.setdefault("OMP_NUM_THREADS", str(cores))
+    import oracle
+
+    outs = {}
+    t_layer = []
+    deadline = time.perf_counter() + reps_target_s
+    while True:
+        t0 = time.perf_counter()
+        for name in SHAPES:
+            W, mask, x = host[name]
+            outs[name] = oracle.linear_bf16(x[:M], W, mask)
+        t_layer.append(time.perf_counter() - t0)
+        if time.perf_counter() > deadline or len(t_layer) >= 5:
+            break
+    t = sorted(t_layer)[len(t_layer) // 2]
+    return ({"value": M / (LAYERS * t), "unit": "tok/s", "cores": cores, "kind": "oracle",
+             "sample": f"layer 0 of {LAYERS} (qkv, o, gate_up, down) at M={M}, float64 C oracle with OpenMP over "
+                       f"output rows, median of {len(t_layer)} runs of {t:.2f} s, scaled x{LAYERS} to one step"},
+            outs)
+
+
+REF_ROW_FRACTION = 8  # each reference step computes 1/8 of every layer-0 output row set
+
+
+def run_reference(args):
+    """The float64 oracle on the host cores, on the same workload: each step computes
+    every 8th output row of the four layer-0 linears (a bounded sample), and the time is
+    scaled by 8 x 32 to a full 32-layer step."""
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    host = host_layer(args.pct, args.m)
+    cores = len(os.sched_getaffinity(0))
+    os.environ.setdefault("OMP_NUM_THREADS", str(cores))
+    import numpy as np
+
+    import oracle
+
+    sample = {}
+    for name in SHAPES:
+        W, mask, x = host[name]
+        rows = np.arange(0, W.shape[0], REF_ROW_FRACTION)
+        sample[name] = (np.ascontiguousarray(W[rows]), np.ascontiguousarray(mask[rows]), x[: args.m])
+
+    def step():
+        for name in SHAPES:
+            W, mask, x = sample[name]
+            oracle.linear_bf16(x, W, mask)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    t = (time.perf_counter() - t0) / args.steps * REF_ROW_FRACTION * LAYERS
+    value = args.m / t
+    line = {"metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, Llama-2-7B shapes)", "impl": "reference",
+            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
+                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
+                                   f"sparsity, bf16 bitmask format, decode M={args.m}", "M": args.m},
+            "cpu_baseline": {"value": value, "unit": "tok/s", "cores": cores, "kind": "oracle",
+                             "sample": f"each step: every {REF_ROW_FRACTION}th output row of the four layer-0 "
+                                       f"linears at M={args.m}; time scaled x{REF_ROW_FRACTION * LAYERS}"},
+            "e2e": {"value": value, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    from paper_2405_03594_gb300 import sp, synth
+
+    Ms = sorted({args.m} | {int(v) for v in args.sweep.split(",") if v.strip()})
+    Mmax = max(Ms)
+    host = host_layer(args.pct, Mmax)
+    mats, xs, ys = {}, {}, {}
+    for name in SHAPES:
+        W, mask, x = host[name]
+        h0 = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
+                         torch.from_numpy(mask).to(dev))
+        mats[name] = [h0] + [h0.clone() for _ in range(LAYERS - 1)]
+        xs[name] = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+        ys[name] = torch.empty((Mmax, h0.n), dtype=torch.bfloat16, device=dev)
+    torch.cuda.synchronize()
+    ws_bytes = max(h.workspace_size(Mmax) for h in (mats[n][0] for n in SHAPES))
+    ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
+
+    def linear(name, layer, M, stream=None):
+        mats[name][layer].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path, stream=stream)
+
+    def per_m(M):
+        # one CUDA graph per shape: its 32 layers back to back
+        for name in SHAPES:
+            linear(name, 0, M)
+        torch.cuda.synchronize()
+        graphs = {}
+        for name in SHAPES:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                for layer in range(LAYERS):
+                    linear(name, layer, M)
+            graphs[name] = g
+        torch.cuda.synchronize()
+        stream = torch.cuda.current_stream()
+        for _ in range(args.warmup):
+            for name in SHAPES:
+                graphs[name].replay()
+        torch.cuda.synchronize()
+        ev = {name: [] for name in SHAPES}
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for _ in range(args.steps):
+            for name in SHAPES:
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                graphs[name].replay()
+                b.record(stream)
+                ev[name].append((a, b))
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        total_ms = t_start.elapsed_time(t_end)
+        shape_ms = {name: sum(a.elapsed_time(b) for a, b in ev[name]) for name in SHAPES}
+        sp.check()
+        return total_ms, shape_ms, graphs
+
+    results = {}
+    peak_gbs, peak_kind = load_peaks()
+    for M in Ms:
+        if M == args.m:
+            with ClockSampler(local_rank) as clk:
+                total_ms, shape_ms, graphs = per_m(M)
+            clocks = clk.summary()
+        else:
+            total_ms, shape_ms, graphs = per_m(M)
+        del graphs
+        step_ms = total_ms / args.steps
+        if world > 1:
+            t = torch.tensor([step_ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            step_ms = float(t.item())
+        step_bytes = 0
+        per_shape = {}
+        for name in SHAPES:
+            h = mats[name][0]
+            b = algorithmic_bytes(h.info, M, h.k, h.n)
+            step_bytes += LAYERS * b
+            launch_us = shape_ms[name] / (args.steps * LAYERS) * 1e3
+            per_shape[name] = {"us_per_launch": launch_us, "algorithmic_bytes": b,
+                               "gbs": b / (launch_us * 1e-6) / 1e9, "frac": b / (launch_us * 1e-6) / 1e9 / peak_gbs}
+        results[M] = {"step_ms": step_ms, "tok_s": world * M / (step_ms * 1e-3),
+                      "step_gbs": step_bytes / (step_ms * 1e-3) / 1e9, "per_shape": per_shape,
+                      "step_bytes": step_bytes}
+
+    M = args.m
+    r = results[M]
+    dom = max(SHAPES, key=lambda n: r["per_shape"][n]["us_per_launch"])
+    d = r["per_shape"][dom]
+    kern = "linear_cc_kernel"
+    workload = f"{dom} {args.pct}% bf16 M={M}"
+    roofline = {"bound": "hbm", "achieved": d["gbs"], "peak": peak_gbs, "unit": "GB/s", "frac": d["frac"],
+                "traffic": profiled_traffic(kern, workload), "kernel": kern, "launch": workload,
+                "peak_kind": f"of {peak_kind} (MEASURED_PEAKS.json hbm_gbs, copy)" if peak_kind == "measured"
+                else "of fallback",
+                "algorithmic_bytes_per_launch": d["algorithmic_bytes"], "us_per_launch": d["us_per_launch"]}
+
+    # ---------------------------------------------------------------- end to end
+    # Public API calls (no graph), inputs copied from pinned host memory every step and
+    # the step's result (the last down projection) copied back.
+    pinned_x = {name: xs[name][:M].cpu().pin_memory() for name in SHAPES}
+    pinned_y = torch.empty((M, mats["down"][0].n), dtype=torch.bfloat16).pin_memory()
+    stream = torch.cuda.current_stream()
+    e2e_steps = max(3, min(args.steps, 50))
+
+    def e2e_step():
+        for name in SHAPES:
+            xs[name][:M].copy_(pinned_x[name], non_blocking=True)
+        for layer in range(LAYERS):
+            for name in SHAPES:
+                linear(name, layer, M)
+        pinned_y.copy_(ys["down"][:M], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = a.elapsed_time(b) / e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    h2d = sum(pinned_x[n].numel() * 2 for n in SHAPES)
+    d2h = pinned_y.numel() * 2
+
+    # ---------------------------------------------------------------- parity + CPU oracle (rank 0, N=1)
+    cpu = None
+    parity = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu, outs = cpu_oracle_leg(host, M)
+        worst = 0.0
+        fro = 0.0
+        for name in SHAPES:
+            mats[name][0].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path)
+            y = synth.bf16_to_f32(ys[name][:M].view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.float64)
+            ref = outs[name]
+            worst = max(worst, float(np.abs(y - ref).max() / np.abs(ref).max()))
+            fro = max(fro, float(np.linalg.norm(y - ref) / np.linalg.norm(ref)))
+        parity = {"max_err_over_max_ref": worst, "rel_fro": fro, "ok": worst <= 1e-2 and fro <= 5e-3}
+
+    if rank == 0:
+        launches_per_step = LAYERS * len(SHAPES) * ((M + 15) // 16)
+        line = {
+            "metric": METRIC, "value": r["tok_s"], "unit": "tok/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded N(0,0.02^2) bf16 weights, per-row magnitude masks, N(0,1) bf16 x; "
+                    "32 device copies of layer 0",
+            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
+                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
+                                   f"sparsity, bf16 bitmask format, decode M={M}",
+                       "M": M, "layers": LAYERS, "sparsity_pct": args.pct, "path": args.path,
+                       "l2": f"no flush: inputs larger than L2 ({r['step_bytes'] / 1e9:.2f} GB of distinct "
+                             f"compressed weights per step)",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "e2e": {"value": world * M / (e2e_ms * 1e-3), "unit": "tok/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "how": "public sp.linear calls (no graph) with pinned host x "
+                                                      "copied in and the last down output copied out per step"},
+            "gpu_launches": launches_per_step * args.steps,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "clocks": clocks,
+            "step_gbs": r["step_gbs"],
+            "parity_layer0": parity,
+            "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
+                               "frac_of_peak": v["step_gbs"] / peak_gbs,
+                               "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),
+                                                 "frac": round(s["frac"], 4)} for n, s in v["per_shape"].items()}}
+                      for m, v in results.items()},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_single(args):
+    """One linear of one shape, launched directly: a small case for ncu captures."""
+    import numpy as np
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+
+    dev = torch.device("cuda", 0)
+    W, mask, x = synth.layer_inputs(args.single, args.pct, args.m, seed=0, layer=0)
+    h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16), torch.from_numpy(mask).to(dev))
+    xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+    y = torch.empty((args.m, h.n), dtype=torch.bfloat16, device=dev)
+    ws = torch.zeros(max(h.workspace_size(args.m), 256), dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        h.linear(xd, out=y, workspace=ws, path=args.path)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        h.linear(xd, out=y, workspace=ws, path=args.path)
+    b.record()
+    torch.cuda.synchronize()
+    sp.check()
+    us = a.elapsed_time(b) / max(args.steps, 1) * 1e3
+    nbytes = algorithmic_bytes(h.info, args.m, h.k, h.n)
+    print(json.dumps({"single": args.single, "M": args.m, "pct": args.pct, "us_per_launch": us,
+                      "algorithmic_bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}), flush=True)
+
+
+def main():
+    args = parse()
+    if args.single:
+        run_single(args)
+        return
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -5,20 +5,22 @@
 // memory onto the chip and are expanded there by their bitmask; decode is bound
 // by those bytes, Sec. 2.4, 3.4).
 //
-// Launch: G persistent CTAs (2 per SM), each owning a contiguous run of chunks in
+// Launch: G persistent CTAs (4 per SM), each owning a contiguous run of chunks in
 // storage order (stream-K), so every CTA streams one linear byte range.
-//   warp 4, lane 0   producer: one cp.async.bulk per chunk (+ one 128-byte copy
-//                    of x[m, 64t : 64t+64) per batch row) into a ring of
-//                    `slots` shared-memory slots, each guarded by a full/empty
-//                    mbarrier pair; weight bytes carry an L2 evict-first hint.
-//   warps 0-3        consumers, thread r <-> row r of the chunk: its value slot
-//                    is a popc prefix sum over the chunk's masks (warp scan plus
-//                    the other warps' redux sums); it walks its set bits, gathers
-//                    x[m, 64t+j] from registers of lane j%32 by shuffle, and
-//                    accumulates in FP32.  At a row-block end the 128 rows are
-//                    written (bf16, RNE), or -- when the row block is shared with
-//                    other CTAs -- stored as an FP32 partial and summed in CTA
-//                    order by the last CTA to arrive (deterministic split-K).
+//   warp 4, lane 0   producer: one cp.async.bulk per chunk (+ one copy of
+//                    x[m, 64t : 64t+64) per batch row) into a ring of `slots`
+//                    shared-memory slots, each guarded by a full/empty mbarrier
+//                    pair; weight bytes carry an L2 evict-first hint.
+//   warps 0-3        consumers, thread r <-> row r of the chunk: its first value is
+//                    found by a popc prefix sum over the chunk's masks (warp scan plus
+//                    the other warps' redux sums); it walks its set bits (two
+//                    independent chains: columns 0-31 and 32-63), gathers
+//                    x[m, 64t+j] from lane j%32 by shuffle (two batch rows per
+//                    register), and accumulates with the FP32-accumulating bf16 FMA.
+//                    At a row-block end the 128 rows are written (bf16, RNE), or --
+//                    when the row block is shared with other CTAs -- stored as an FP32
+//                    partial and summed in CTA order by the last CTA to arrive
+//                    (deterministic split-K).
 #include <algorithm>
 
 #include "sp_internal.cuh"
@@ -28,13 +30,47 @@ namespace {
 
 constexpr int kConsumerWarps = 4;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;
-constexpr int kMaxTokens = 8;  // batch rows per launch of this kernel
+constexpr int kMaxTokens = 16;  // batch rows per launch of this kernel
 constexpr int kMaxDevices = 64;
-constexpr size_t kSmemBudget = 110 * 1024;  // ring slots; two CTAs share one SM
-constexpr size_t kSmemOptIn = 112 * 1024;
+constexpr int kCtasPerSm = 4;
+constexpr size_t kSmemBudget = 53 * 1024;  // ring slots per CTA; four CTAs share one SM
+constexpr size_t kSmemOptIn = 54 * 1024;
+
+// Index of the most significant set bit, or -1 for 0.
+__device__ __forceinline__ int msb32(uint32_t v) {
+  int r;
+  asm("bfind.u32 %0, %1;" : "=r"(r) : "r"(v));
+  return r;
+}
+// 1 << j for j in [0, 31]; 0 for j = -1 (PTX clamps the shift amount).
+__device__ __forceinline__ uint32_t bit32(int j) {
+  uint32_t r;
+  asm("shl.b32 %0, 1, %1;" : "=r"(r) : "r"(j));
+  return r;
+}
+// acc + a * b with bf16 a, b and an FP32 accumulator (sm_100+ mixed-precision FMA).
+__device__ __forceinline__ float fma_bf16(uint16_t a, uint16_t b, float c) {
+  float d;
+  asm("fma.rn.f32.bf16 %0, %1, %2, %3;" : "=f"(d) : "h"(a), "h"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ uint16_t lo16(uint32_t v) { return (uint16_t)(v & 0xffffu); }
+__device__ __forceinline__ uint16_t hi16(uint32_t v) { return (uint16_t)(v >> 16); }
+// int8 weight -> bf16 bits, exact for |q| <= 128: the byte lands in the mantissa of
+// 2^23 + 128 + q, the float subtraction leaves q, and q fits bf16's 8-bit significand.
+__device__ __forceinline__ uint16_t i8_to_bf16(uint32_t byte) {
+  const float f = __uint_as_float(0x4B000000u | (byte ^ 0x80u)) - 8388736.0f;
+  return (uint16_t)(__float_as_uint(f) >> 16);
+}
+
+template <int ES>
+__device__ __forceinline__ uint16_t load_w(const uint8_t* vals, int idx) {
+  if (ES == 2) return reinterpret_cast<const uint16_t*>(vals)[idx];
+  return i8_to_bf16(vals[idx]);
+}
 
 template <int M, int ES>
-__global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearParams p) {
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
@@ -43,9 +79,10 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
   const int64_t w0 = range_begin(blockIdx.x, p.W, p.G);
   const int64_t w1 = range_begin(blockIdx.x + 1, p.W, p.G);
   const int T = p.T;
+  const int slots = p.slots;
 
   if (tid == 0) {
-    for (int s = 0; s < p.slots; ++s) {
+    for (int s = 0; s < slots; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kConsumerWarps);
     }
@@ -56,41 +93,74 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
   if (warp == kConsumerWarps) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+      // Weight bytes do not depend on the previous kernel in the stream: the first
+      // ring fill is issued before griddepcontrol.wait; every x copy comes after it.
       const uint64_t pol = policy_evict_first();
-      int64_t it = 0;
-      for (int64_t w = w0; w < w1; ++w, ++it) {
-        const int s = (int)(it % p.slots);
-        const uint32_t ph = (uint32_t)((it / p.slots) & 1);
-        if (it >= p.slots && !mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
-          set_status(p.status, kStatusTimeout);
-          break;
+      const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
+      {
+        int t = (int)(w0 % T);
+        for (int64_t i = 0; i < n_pre; ++i) {
+          const int64_t w = w0 + i;
+          const uint64_t o0 = p.off[w];
+          const uint32_t bytes = (uint32_t)(p.off[w + 1] - o0);
+          const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
+          mbar_arrive_expect_tx(&full[i], bytes + (uint32_t)M * (uint32_t)valid * 2u);
+          bulk_g2s_hint(smem + (size_t)i * p.slot_bytes, p.buf + o0, bytes, &full[i], pol);
+          if (++t == T) t = 0;
         }
-        const int t = (int)(w % T);
-        const uint64_t o0 = p.off[w];
-        const uint32_t bytes = (uint32_t)(p.off[w + 1] - o0);
+      }
+      pdl_wait();
+      pdl_launch_dependents();
+      int s = 0;
+      uint32_t ph = 0;
+      int t = (int)(w0 % T);
+      int64_t n_issued = 0;
+      for (int64_t w = w0; w < w1; ++w, ++n_issued) {
         const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
         const uint32_t xb = (uint32_t)valid * 2u;
         uint8_t* slot = smem + (size_t)s * p.slot_bytes;
-        mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
-        bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
+        if (n_issued >= n_pre) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+            set_status(p.status, kStatusTimeout);
+            break;
+          }
+          const uint64_t o0 = p.off[w];
+          const uint32_t bytes = (uint32_t)(p.off[w + 1] - o0);
+          mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
+          bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
+        }
 #pragma unroll
         for (int m = 0; m < M; ++m)
           bulk_g2s(slot + p.chunk_region + m * 128, p.x + (int64_t)m * p.K + (int64_t)kTileK * t, xb, &full[s]);
+        if (++t == T) t = 0;
+        if (++s == slots) {
+          s = 0;
+          ph ^= 1u;
+        }
       }
     }
     return;
   }
 
   // -------------------------------------------------------------- consumers
+  pdl_wait();  // y, the workspace and x belong to the stream order
+  pdl_launch_dependents();
+  // Thread r owns row r of every chunk.  Its 64-bit mask splits into two 32-column
+  // halves walked as two independent chains, each from its highest set bit down
+  // (bfind), consuming that half's values from the top.  Lane j holds x[m, 64t+j]
+  // (low half) and x[m, 64t+32+j] (high half), two batch rows per register, and the
+  // other lanes fetch them by shuffle.
+  constexpr int MP = (M + 1) / 2;
   float acc[M];
 #pragma unroll
   for (int m = 0; m < M; ++m) acc[m] = 0.f;
   bool dead = false;  // a bounded wait expired: keep the barrier schedule, skip the math
   const int64_t rb_first = w0 / T;
-  int64_t it = 0;
-  for (int64_t w = w0; w < w1; ++w, ++it) {
-    const int s = (int)(it % p.slots);
-    const uint32_t ph = (uint32_t)((it / p.slots) & 1);
+  int64_t rb = rb_first;
+  int t = (int)(w0 % T);
+  int s = 0;
+  uint32_t ph = 0;
+  for (int64_t w = w0; w < w1; ++w) {
     if (!dead) {
       // the decision must be warp-uniform: the shuffles below use the full mask
       const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
@@ -102,8 +172,9 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
     if (!dead) {
       const uint8_t* slot = smem + (size_t)s * p.slot_bytes;
       const uint64_t* masks = reinterpret_cast<const uint64_t*>(slot);
-      uint64_t mk = masks[tid];
-      const int pc = __popcll(mk);
+      const uint64_t mk = masks[tid];
+      uint32_t lo = (uint32_t)mk, hi = (uint32_t)(mk >> 32);
+      const int plo = __popc(lo), pc = plo + __popc(hi);
       int incl = pc;
 #pragma unroll
       for (int d = 1; d < 32; d <<= 1) {
@@ -115,50 +186,68 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
       const int e0 = base + incl - pc;
 
       const uint16_t* xs = reinterpret_cast<const uint16_t*>(slot + p.chunk_region);
-      uint32_t xr[M];
+      uint32_t XL[MP], XH[MP];
 #pragma unroll
-      for (int m = 0; m < M; ++m) xr[m] = (uint32_t)xs[m * 64 + lane] | ((uint32_t)xs[m * 64 + 32 + lane] << 16);
-
-      const uint8_t* vals = slot + kMaskBytes + (size_t)e0 * ES;
-      const int iters = (int)__reduce_max_sync(0xffffffffu, (unsigned)pc);
+      for (int q = 0; q < MP; ++q) {
+        const uint32_t a0 = xs[(2 * q) * 64 + lane], b0 = xs[(2 * q) * 64 + 32 + lane];
+        const uint32_t a1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + lane] : 0u;
+        const uint32_t b1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + 32 + lane] : 0u;
+        XL[q] = a0 | (a1 << 16);
+        XH[q] = b0 | (b1 << 16);
+      }
+      const uint8_t* vals = slot + kMaskBytes;
+      const int top_lo = e0 + plo - 1;  // highest-column value of the low half
+      const int top_hi = e0 + pc - 1;   // ... of the high half
+      const int iters = (int)__reduce_max_sync(0xffffffffu, (unsigned)max(plo, pc - plo));
+#pragma unroll 2
       for (int q = 0; q < iters; ++q) {
-        const bool act = mk != 0;
-        const int j = act ? (__ffsll((long long)mk) - 1) : 0;
-        mk &= mk - 1;
-        float wv = 0.f;
-        if (act) {
-          if (ES == 2)
-            wv = bf16_bits_to_float(reinterpret_cast<const uint16_t*>(vals)[q]);
-          else
-            wv = (float)reinterpret_cast<const int8_t*>(vals)[q];
-        }
-        const int src = j & 31;
-        const bool hi = j >= 32;
+        const int jl = msb32(lo), jh = msb32(hi);
+        lo &= ~bit32(jl);
+        hi &= ~bit32(jh);
+        const bool al = jl >= 0, ah = jh >= 0;
+        uint16_t wl = 0, wh = 0;
+        if (al) wl = load_w<ES>(vals, top_lo - q);
+        if (ah) wh = load_w<ES>(vals, top_hi - q);
 #pragma unroll
-        for (int m = 0; m < M; ++m) {
-          const uint32_t v = __shfl_sync(0xffffffffu, xr[m], src);
-          const float xv = __uint_as_float(hi ? (v & 0xffff0000u) : (v << 16));
-          if (act) acc[m] = fmaf(wv, xv, acc[m]);
+        for (int r = 0; r < MP; ++r) {
+          const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+          const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+          if (al) {
+            acc[2 * r] = fma_bf16(wl, lo16(xl), acc[2 * r]);
+            if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wl, hi16(xl), acc[2 * r + 1]);
+          }
+          if (ah) {
+            acc[2 * r] = fma_bf16(wh, lo16(xh), acc[2 * r]);
+            if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wh, hi16(xh), acc[2 * r + 1]);
+          }
         }
       }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);
+    if (++s == slots) {
+      s = 0;
+      ph ^= 1u;
+    }
 
     // ------------------------------------------------------------ row-block end
-    const int64_t rb = w / T;
-    const int t = (int)(w % T);
-    if (t != T - 1 && w + 1 != w1) continue;
-    const int64_t seg_begin = rb * T;
-    const int64_t n = rb * kRows + tid;
+    const int t_cur = t;
+    const int64_t rb_cur = rb;
+    if (++t == T) {
+      t = 0;
+      ++rb;
+    }
+    if (t_cur != T - 1 && w + 1 != w1) continue;
+    const int64_t seg_begin = rb_cur * T;
+    const int64_t n = rb_cur * kRows + tid;
     const float sc = (ES == 1 && n < p.N) ? p.scale[n] : 1.f;
-    if (seg_begin >= w0 && t == T - 1) {
+    if (seg_begin >= w0 && t_cur == T - 1) {
       if (n < p.N) {
 #pragma unroll
         for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(acc[m] * sc);
       }
     } else {
-      const int my_slot = (rb == rb_first) ? 0 : 1;
+      const int my_slot = (rb_cur == rb_first) ? 0 : 1;
       float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * (kRows * kMaxTokens);
 #pragma unroll
       for (int m = 0; m < M; ++m) __stcg(wsp + m * kRows + tid, acc[m]);
@@ -166,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
       named_bar_sync(1, kConsumerWarps * 32);
       const int64_t i_first = owner_of(seg_begin, p.W, p.G);
       const int64_t i_last = owner_of(seg_begin + T - 1, p.W, p.G);
-      const int sf = (range_begin(i_first, p.W, p.G) / T == rb) ? 0 : 1;
+      const int sf = (range_begin(i_first, p.W, p.G) / T == rb_cur) ? 0 : 1;
       int* ctr = p.cnt + i_first * 2 + sf;
       if (tid == 0) {
         const int old = atomicAdd(ctr, 1);
@@ -179,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 2) linear_cc_kernel(const LinearPara
 #pragma unroll
         for (int m = 0; m < M; ++m) sum[m] = 0.f;
         for (int64_t i = i_first; i <= i_last; ++i) {
-          const int sl = (range_begin(i, p.W, p.G) / T == rb) ? 0 : 1;
+          const int sl = (range_begin(i, p.W, p.G) / T == rb_cur) ? 0 : 1;
           const float* src = p.ws + (i * 2 + sl) * (kRows * kMaxTokens);
 #pragma unroll
           for (int m = 0; m < M; ++m) sum[m] += __ldcg(src + m * kRows + tid);
@@ -209,7 +298,20 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem) {
       return SP_ERR_CUDA;
     configured[dev] = true;
   }
-  kern<<<p.G, kThreads, smem, stream>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)p.G);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, kern, p) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
   return cudaGetLastError() == cudaSuccess ? SP_OK : SP_ERR_CUDA;
 }
 
@@ -224,14 +326,24 @@ sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem) {
     case 6: return launch_one<6, ES>(p, stream, smem);
     case 7: return launch_one<7, ES>(p, stream, smem);
     case 8: return launch_one<8, ES>(p, stream, smem);
+    case 9: return launch_one<9, ES>(p, stream, smem);
+    case 10: return launch_one<10, ES>(p, stream, smem);
+    case 11: return launch_one<11, ES>(p, stream, smem);
+    case 12: return launch_one<12, ES>(p, stream, smem);
+    case 13: return launch_one<13, ES>(p, stream, smem);
+    case 14: return launch_one<14, ES>(p, stream, smem);
+    case 15: return launch_one<15, ES>(p, stream, smem);
+    case 16: return launch_one<16, ES>(p, stream, smem);
     default: return SP_ERR_INVALID_ARG;
   }
 }
 
 int grid_cc(const sp_matrix* h) {
   const int64_t W = (int64_t)h->RB * h->T;
-  static_assert(2 <= kMaxGridPerSm, "grid must fit the workspace counter region");
-  return (int)std::min<int64_t>((int64_t)2 * h->num_sms, W);
+  static_assert(kCtasPerSm <= kMaxGridPerSm, "grid must fit the workspace counter region");
+  // at least ~6 chunks per CTA, whole multiples of the SM count while W allows
+  const int64_t per_sm = std::max<int64_t>(1, std::min<int64_t>(kCtasPerSm, W / ((int64_t)h->num_sms * 6)));
+  return (int)std::min<int64_t>(per_sm * h->num_sms, W);
 }
 
 }  // namespace

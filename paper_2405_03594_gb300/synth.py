@@ -63,14 +63,31 @@ def n_pruned(pct: int, K: int) -> int:
     return round_half_even_div(pct * K, 100)
 
 
+def _normal_bf16(shape, g: np.random.Generator, std: float | None) -> np.ndarray:
+    """bf16 bits of std * N(0, 1) (or N(0, 1)), drawn row-chunk by row-chunk; the
+    generator's stream is the same as one draw of the full shape."""
+    N, K = shape
+    out = np.empty((N, K), dtype=np.uint16)
+    rows = max(1, (1 << 22) // max(K, 1))
+    buf = np.empty((rows, K), dtype=np.float32)
+    for r0 in range(0, N, rows):
+        r1 = min(N, r0 + rows)
+        b = buf[: r1 - r0]
+        g.standard_normal(out=b, dtype=np.float32)
+        if std is not None:
+            b *= np.float32(std)
+        out[r0:r1] = bf16_from_f32(b)
+    return out
+
+
 def weight(N: int, K: int, g: np.random.Generator, std: float = 0.02) -> np.ndarray:
     """bf16 bits of W ~ N(0, std^2), shape [N, K]."""
-    return bf16_from_f32(g.standard_normal((N, K), dtype=np.float32) * np.float32(std))
+    return _normal_bf16((N, K), g, std)
 
 
 def activations(M: int, K: int, g: np.random.Generator) -> np.ndarray:
     """bf16 bits of x ~ N(0, 1), shape [M, K]."""
-    return bf16_from_f32(g.standard_normal((M, K), dtype=np.float32))
+    return _normal_bf16((M, K), g, None)
 
 
 def _prune_smallest(W: np.ndarray, n_prune_per_row: np.ndarray, keep_cols=None) -> np.ndarray:
@@ -80,22 +97,32 @@ def _prune_smallest(W: np.ndarray, n_prune_per_row: np.ndarray, keep_cols=None) 
     keys are exactly the first n entries of a stable sort on |w|."""
     N, K = W.shape
     assert K < (1 << 20)
-    key = (np.ascontiguousarray(W, dtype=np.uint16) & np.uint16(0x7FFF)).astype(np.uint64)
-    key <<= np.uint64(20)
-    key |= np.arange(K, dtype=np.uint64)[None, :]
+    W = np.ascontiguousarray(W, dtype=np.uint16)
+    n_prune_per_row = np.asarray(n_prune_per_row, dtype=np.int64)
+    cols = np.arange(K, dtype=np.uint64)[None, :]
     if keep_cols is not None:
-        key[:, keep_cols] |= np.uint64(1) << np.uint64(40)  # after every prunable column
+        cols = cols.copy()
+        cols[:, keep_cols] |= np.uint64(1) << np.uint64(40)  # after every prunable column
     mask = np.ones((N, K), dtype=np.uint8)
-    for n in np.unique(n_prune_per_row):
-        rows = np.nonzero(n_prune_per_row == n)[0]
-        if n <= 0:
-            continue
-        if n >= K:
-            mask[rows] = 0
-            continue
-        sub = key[rows]
-        thr = np.partition(sub, n - 1, axis=1)[:, n - 1]
-        mask[rows] = (sub > thr[:, None]).astype(np.uint8)
+    rows_per = max(1, (1 << 21) // K)
+    key = np.empty((rows_per, K), dtype=np.uint64)
+    for r0 in range(0, N, rows_per):
+        r1 = min(N, r0 + rows_per)
+        kk = key[: r1 - r0]
+        np.bitwise_and(W[r0:r1], np.uint16(0x7FFF), out=kk, casting="unsafe")
+        kk <<= np.uint64(20)
+        kk |= cols
+        npr = n_prune_per_row[r0:r1]
+        for n in np.unique(npr):
+            if n <= 0:
+                continue
+            sel = np.nonzero(npr == n)[0]
+            if n >= K:
+                mask[r0 + sel] = 0
+                continue
+            sub = kk if sel.size == kk.shape[0] else kk[sel]
+            thr = np.partition(sub, n - 1, axis=1)[:, n - 1]
+            mask[r0 + sel] = sub > thr[:, None]
     return mask
 
 
