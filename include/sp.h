@@ -125,6 +125,23 @@ sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_de
 sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
                        size_t workspace_bytes, sp_path path, void* stream);
 
+/* sp_linear for callers that may not allocate device memory (the paper has no
+ * counterpart; this is a deployment convenience).  Some callers receive only their
+ * input and output buffers from a host framework or plugin interface that owns all
+ * device memory, and some run latency-critical loops where cudaMalloc/cudaFree would
+ * synchronise the device: neither can supply sp_linear's workspace.  This call runs the
+ * same CUDA-core decode kernel with the same launch configuration, using instead a
+ * scratch array of 16 MiB that the library keeps on every GPU that loads it (held until
+ * the process exits).  It calls no cudaMalloc, cudaFree or other allocating routine.
+ *   x_dev [m, K] bf16, y_dev [m, N] bf16, as for sp_linear.
+ *   Returns SP_ERR_WORKSPACE if the kernel would need more scratch than the array holds.
+ *   The first call on a device looks up the array's device address (set-up, once per
+ *   device, with that device current); make that first call before any stream capture.
+ *   Every call on a device shares the one array, and a call clears its arrival counters
+ *   first: calls that overlap on the GPU (other streams, other threads) race and give
+ *   wrong results; order them on one stream. */
+sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* stream);
+
 /* A copy of the handle with its own device buffers (same bytes). */
 sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx, void* stream,
                    sp_matrix** out);

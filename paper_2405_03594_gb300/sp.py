@@ -24,8 +24,8 @@ STATUS = {
     5: "SP_ERR_OUT_OF_MEMORY", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_BAD_HANDLE", 8: "SP_ERR_WORKSPACE",
 }
 # every function declared in include/sp.h
-EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_clone", "sp_free",
-           "sp_info", "sp_copy_out", "sp_check", "sp_status_string"]
+EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_linear_noalloc",
+           "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string"]
 
 
 class SpError(RuntimeError):
@@ -55,6 +55,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_workspace_size.argtypes = [P, I64, ctypes.POINTER(SZ)]
     lib.sp_linear.argtypes = [P, P, I64, P, P, SZ, P]
     lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
+    lib.sp_linear_noalloc.argtypes = [P, P, I64, P, P]
     lib.sp_clone.argtypes = [P, ALLOC_FN, FREE_FN, P, P, ctypes.POINTER(P)]
     lib.sp_free.argtypes = [P]
     lib.sp_info.argtypes = [P, ctypes.POINTER(SpInfo)]
@@ -140,6 +141,14 @@ class SparseMatrix:
             workspace = workspace_for(self.workspace_size(m), x.device)
         _check(_lib.sp_linear_ex(self._h, _ptr(x), m, _ptr(out), _ptr(workspace), workspace.numel(), PATHS[path],
                                  _stream(stream)), "sp_linear")
+        return out
+
+    def linear_noalloc(self, x: torch.Tensor, out: torch.Tensor, stream=None) -> torch.Tensor:
+        """sp_linear_noalloc: the decode kernel with the library's own static scratch, for
+        callers that cannot allocate device memory; `out` [m, N] bf16 must be given."""
+        assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
+        assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
+        _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)), "sp_linear_noalloc")
         return out
 
     def decompress(self, stream=None) -> torch.Tensor:
