@@ -21,8 +21,9 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 bool live(const sp_matrix* h) { return h && h->magic == SP_MAGIC; }
 
-// Largest batch that the CUDA-core family takes under SP_PATH_AUTO.
-constexpr int64_t kCudaCoreMaxM = 1 << 30;
+// Largest batch that the CUDA-core family takes under SP_PATH_AUTO; larger batches go
+// to the tensor-core family.
+constexpr int64_t kCudaCoreMaxM = 16;
 }  // namespace
 
 int* device_status_ptr() {
@@ -98,7 +99,7 @@ sp_status sp_decompress(const sp_matrix* h, void* w_out_dev, void* stream) {
 sp_status sp_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes) {
   if (!live(h)) return SP_ERR_BAD_HANDLE;
   if (!bytes || m < 0) return SP_ERR_INVALID_ARG;
-  *bytes = m == 0 ? 0 : workspace_bytes_cc(h, m);
+  *bytes = m == 0 ? 0 : std::max(workspace_bytes_cc(h, m), workspace_bytes_tc(h, m));
   return SP_OK;
 }
 
@@ -116,8 +117,9 @@ sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y
     return SP_ERR_CUDA;
   }
   if (dev != h->device) return SP_ERR_INVALID_ARG;
-  if (path == SP_PATH_TENSOR_CORE) return SP_ERR_UNSUPPORTED;
-  if (path == SP_PATH_AUTO && m > kCudaCoreMaxM) return SP_ERR_UNSUPPORTED;
+  if (path == SP_PATH_TENSOR_CORE || (path == SP_PATH_AUTO && m > kCudaCoreMaxM))
+    return launch_linear_tc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
+                            workspace_bytes, (cudaStream_t)stream);
   return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
                           workspace_bytes, (cudaStream_t)stream);
 }

@@ -166,6 +166,9 @@ sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
+sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
+                           cudaStream_t stream);
+size_t workspace_bytes_tc(const sp_matrix* h, int64_t M);
 int* device_status_ptr();            // this device's status word (device address)
 uint64_t wait_timeout_ns();          // bounded-wait limit for kernels
 void* dev_alloc(const sp_matrix* h, size_t bytes);

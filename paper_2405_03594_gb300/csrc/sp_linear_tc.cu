@@ -1,0 +1,579 @@
+// sp_linear_tc.cu -- sparse linear on the 5th-generation tensor cores (tcgen05).
+//
+// The GPU engine of Sec. 2.4.2: compressed submatrices move from global memory onto
+// the chip, are expanded by their bitmask, and the tensor cores run on the expanded
+// tiles at the dense rate while global traffic stays at the compressed size.  On
+// sm_103a the expanded tile goes to tensor memory and feeds tcgen05.mma directly:
+//
+//   D[128 rows, Ntok tokens] (fp32, TMEM) += A[128 rows, 64 k] (bf16, TMEM) x B[64 k, Ntok]
+//
+// where A is one chunk (128 weight rows x one 64-wide K-tile) expanded by its masks and
+// B is x[tokens, 64t : 64t+64) brought in by TMA (128-byte swizzle, K-major).
+//
+// CTA (one per SM, persistent, stream-K over work items (token tile, row block, K-tile)):
+//   warp 0 lane 0   producer: cp.async.bulk of each chunk and a TMA tile of x into a
+//                   ring of shared-memory slots (full/empty mbarriers);
+//   warp 1          TMEM allocation; lane 0 issues the MMAs (4 x K=16 per chunk) and
+//                   commits them to mbarriers that free A stages, ring slots and D;
+//   warps 2-9       two expander warpgroups taking alternate chunks: thread r of a
+//                   warpgroup owns TMEM lane / chunk row r; it finds its first value by a
+//                   popc prefix sum, expands 64 columns into 32 bf16x2 registers, and
+//                   stores them to an A stage with tcgen05.st; at a row-block end the
+//                   warpgroup that expanded the last K-tile reads D with tcgen05.ld and
+//                   writes bf16 y (RNE), or an FP32 partial for the deterministic
+//                   stream-K fix-up shared with the CUDA-core kernel.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "sp_internal.cuh"
+
+namespace sp {
+namespace {
+
+constexpr int kExpGroups = 2;         // expander warpgroups, taking alternate chunks
+constexpr int kThreads = (2 + 4 * kExpGroups) * 32;
+constexpr int kExpWarp0 = 2;          // first expander warp
+constexpr int kAStages = 4;           // A tiles in TMEM
+constexpr int kMaxNtok = 256;         // tokens per tile (MMA N)
+constexpr uint32_t kTmemCols = 512;   // D (<= 256 columns) + kAStages x 32 columns
+constexpr uint32_t kACol0 = 256;
+constexpr size_t kSmemLimit = 226 * 1024;
+constexpr int kMaxDevices = 64;
+constexpr int kMaxSlots = 16;
+
+// ------------------------------------------------------------------ tcgen05 / TMA wrappers
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_store32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+      "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]),
+      "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]),
+      "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_store_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_load32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_load_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// D[tmem] (+)= A[tmem] * B[smem desc]; bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void mma_ts(uint32_t d_taddr, uint32_t a_taddr, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_taddr),
+      "r"(a_taddr), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row atoms of
+// 1024 bytes stacked along M/N (stride byte offset 1024), atom base 1024-byte aligned.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);        // start address
+  d |= (uint64_t)1u << 16;                        // leading byte offset (unused for SW128 K-major)
+  d |= (uint64_t)((1024u >> 4) & 0x3FFFu) << 32;  // stride byte offset
+  d |= (uint64_t)1u << 46;                        // descriptor version (sm_100 family)
+  d |= (uint64_t)2u << 61;                        // swizzle mode: 128B
+  return d;
+}
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major, M = 128.
+__host__ __device__ constexpr uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
+__device__ __forceinline__ uint16_t i8_to_bf16(uint32_t byte) {
+  const float f = __uint_as_float(0x4B000000u | (byte ^ 0x80u)) - 8388736.0f;
+  return (uint16_t)(__float_as_uint(f) >> 16);
+}
+
+struct TcParams {
+  LinearParams p;     // shared fields (buf, off, scale, y, ws, cnt, status, N, K, T, RB, M, W, G, slots, ...)
+  int32_t ntok;       // tokens per tile (MMA N), multiple of 16, <= 256
+  int32_t mt;         // token tiles
+  uint32_t b_bytes;   // bytes of one x tile in shared memory (ntok * 128)
+  uint32_t chunk_off; // offset of the chunk region inside a slot
+};
+
+template <int ES>
+__global__ void __launch_bounds__(kThreads, 1)
+    linear_tc_kernel(const __grid_constant__ TcParams tp, const __grid_constant__ CUtensorMap tmap_x) {
+  extern __shared__ uint8_t smem_raw[];
+  const LinearParams& p = tp.p;
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const int slots = p.slots;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)slots * p.slot_bytes);
+  uint64_t* empty = full + slots;
+  uint64_t* a_full = empty + slots;
+  uint64_t* a_empty = a_full + kAStages;
+  // D handshakes, one pair per expander warpgroup: a group's epilogues are sequential,
+  // so each group's parity waits never alias an older phase.
+  uint64_t* d_full = a_empty + kAStages;   // [kExpGroups]
+  uint64_t* d_empty = d_full + kExpGroups; // [kExpGroups]
+  uint32_t* tmem_base_slot = reinterpret_cast<uint32_t*>(d_empty + kExpGroups);
+  volatile int* s_flag = reinterpret_cast<volatile int*>(tmem_base_slot + 1);  // one per warpgroup
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t w0 = range_begin(blockIdx.x, p.W, p.G);
+  const int64_t w1 = range_begin(blockIdx.x + 1, p.W, p.G);
+  const int T = p.T;
+  const int64_t C = (int64_t)p.RB * T;  // chunks per token tile
+
+  if (tid == 0) {
+    for (int s = 0; s < slots; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 4 + 1);  // four expander warps + one MMA commit
+    }
+    for (int a = 0; a < kAStages; ++a) {
+      mbar_init(&a_full[a], 4);
+      mbar_init(&a_empty[a], 1);
+    }
+    for (int g = 0; g < kExpGroups; ++g) {
+      mbar_init(&d_full[g], 1);
+      mbar_init(&d_empty[g], 4);
+    }
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_base_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == 0 && lane == 0) prefetch_tmap(&tmap_x);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_base_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
+      for (int64_t i = 0; i < n_pre; ++i) {  // weight bytes do not depend on the previous grid
+        const int64_t c = (w0 + i) % C;
+        const uint64_t o0 = p.off[c];
+        const uint32_t bytes = (uint32_t)(p.off[c + 1] - o0);
+        mbar_arrive_expect_tx(&full[i], bytes + tp.b_bytes);
+        bulk_g2s_hint(smem + (size_t)i * p.slot_bytes + tp.chunk_off, p.buf + o0, bytes, &full[i], pol);
+      }
+      pdl_wait();
+      pdl_launch_dependents();
+      int s = 0;
+      uint32_t ph = 0;
+      for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
+        const int64_t mtile = w / C;
+        const int64_t c = w % C;
+        const int t = (int)(c % T);
+        uint8_t* slot = smem + (size_t)s * p.slot_bytes;
+        if (n >= n_pre) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+            set_status(p.status, kStatusTimeout);
+            break;
+          }
+          const uint64_t o0 = p.off[c];
+          const uint32_t bytes = (uint32_t)(p.off[c + 1] - o0);
+          mbar_arrive_expect_tx(&full[s], bytes + tp.b_bytes);
+          bulk_g2s_hint(slot + tp.chunk_off, p.buf + o0, bytes, &full[s], pol);
+        }
+        tma_load_2d(slot, &tmap_x, kTileK * t, (int)(mtile * tp.ntok), &full[s]);
+        if (++s == slots) {
+          s = 0;
+          ph ^= 1u;
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      pdl_wait();
+      pdl_launch_dependents();
+      const uint32_t idesc = idesc_bf16(tp.ntok);
+      int s = 0, as = 0;
+      uint32_t ph = 0, aph = 0;
+      uint32_t dph[kExpGroups] = {};
+      int prev_group = -1;  // warpgroup that ran the previous segment's epilogue
+      bool dead = false;
+      for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
+        const bool seg_first = (w == w0) || (w % T == 0);
+        const bool seg_last = (w + 1 == w1) || ((w + 1) % T == 0);
+        if (!dead && seg_first && prev_group >= 0) {
+          // D is reused: wait until that epilogue has read the previous segment
+          if (!mbar_wait(&d_empty[prev_group], dph[prev_group], p.timeout_ns)) {
+            dead = true;
+            set_status(p.status, kStatusTimeout);
+          }
+          dph[prev_group] ^= 1u;
+        }
+        if (!dead && !mbar_wait(&full[s], ph, p.timeout_ns)) {
+          dead = true;
+          set_status(p.status, kStatusTimeout);
+        }
+        if (!dead && !mbar_wait(&a_full[as], aph, p.timeout_ns)) {
+          dead = true;
+          set_status(p.status, kStatusTimeout);
+        }
+        if (!dead) {
+          tc_fence_after();
+          const uint32_t b_saddr = smem_u32(smem + (size_t)s * p.slot_bytes);
+          const uint32_t a_taddr = tmem + kACol0 + (uint32_t)as * 32u;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t bdesc = smem_desc_sw128(b_saddr + (uint32_t)kk * 32u);
+            mma_ts(tmem, a_taddr + (uint32_t)kk * 8u, bdesc, idesc, (seg_first && kk == 0) ? 0u : 1u);
+          }
+          mma_commit(&empty[s]);
+          mma_commit(&a_empty[as]);
+          if (seg_last) mma_commit(&d_full[n % kExpGroups]);
+        }
+        if (seg_last) prev_group = (int)(n % kExpGroups);
+        if (++s == slots) {
+          s = 0;
+          ph ^= 1u;
+        }
+        if (++as == kAStages) {
+          as = 0;
+          aph ^= 1u;
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ expanders + epilogue
+    pdl_wait();
+    pdl_launch_dependents();
+    const int grp = (warp - kExpWarp0) >> 2;  // this warpgroup takes items n = grp (mod 2)
+    const int q = warp & 3;                   // TMEM lane quarter this warp may access
+    const int r = q * 32 + lane;              // chunk row == TMEM lane
+    const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+    const int tid128 = (warp - kExpWarp0 - 4 * grp) * 32 + lane;
+    bool dead = false;
+    uint32_t dph = 0;  // phase of this group's own D handshake
+    const int64_t sg_first = w0 / T;
+    for (int64_t w = w0 + grp, n = grp; w < w1; w += kExpGroups, n += kExpGroups) {
+      const int s = (int)(n % slots);
+      const uint32_t ph = (uint32_t)((n / slots) & 1);
+      const int as = (int)(n % kAStages);
+      const uint32_t aph = (uint32_t)((n / kAStages) & 1);
+      if (!dead) {
+        bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
+        if (ok && n >= kAStages) ok = __all_sync(0xffffffffu, mbar_wait(&a_empty[as], aph ^ 1u, p.timeout_ns));
+        if (!ok) {
+          dead = true;
+          set_status(p.status, kStatusTimeout);
+        }
+      }
+      if (!dead) {
+        tc_fence_after();
+        const uint8_t* chunk = smem + (size_t)s * p.slot_bytes + tp.chunk_off;
+        const uint64_t* masks = reinterpret_cast<const uint64_t*>(chunk);
+        const uint64_t mk = masks[r];
+        const uint32_t mlo = (uint32_t)mk, mhi = (uint32_t)(mk >> 32);
+        const int plo = __popc(mlo);
+        const int pc = plo + __popc(mhi);
+        int incl = pc;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+          const int u = __shfl_up_sync(0xffffffffu, incl, d);
+          if (lane >= d) incl += u;
+        }
+        int base = 0;
+        for (int k = 0; k < q; ++k) base += (int)__reduce_add_sync(0xffffffffu, __popcll(masks[lane + 32 * k]));
+        const int e0 = base + incl - pc;
+        // Static walk over the 64 columns: a kept column takes the next value of its
+        // half's stream.  Columns 0-31 and 32-63 read two independent streams (the
+        // second starts after the first half's plo values) for instruction-level
+        // parallelism; each step is one predicate-setting AND, a predicated load and a
+        // predicated pointer increment.
+        uint32_t o[32];
+        if (ES == 2) {
+          const uint16_t* va = reinterpret_cast<const uint16_t*>(chunk + kMaskBytes) + e0;
+          const uint16_t* vb = va + plo;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            uint32_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;
+            if (mlo & (1u << (2 * i))) a0 = *va++;
+            if (mhi & (1u << (2 * i))) b0 = *vb++;
+            if (mlo & (1u << (2 * i + 1))) a1 = *va++;
+            if (mhi & (1u << (2 * i + 1))) b1 = *vb++;
+            o[i] = __byte_perm(a0, a1, 0x5410);
+            o[16 + i] = __byte_perm(b0, b1, 0x5410);
+          }
+        } else {
+          const uint8_t* va = chunk + kMaskBytes + e0;
+          const uint8_t* vb = va + plo;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            uint32_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;
+            if (mlo & (1u << (2 * i))) a0 = i8_to_bf16(*va++);
+            if (mhi & (1u << (2 * i))) b0 = i8_to_bf16(*vb++);
+            if (mlo & (1u << (2 * i + 1))) a1 = i8_to_bf16(*va++);
+            if (mhi & (1u << (2 * i + 1))) b1 = i8_to_bf16(*vb++);
+            o[i] = __byte_perm(a0, a1, 0x5410);
+            o[16 + i] = __byte_perm(b0, b1, 0x5410);
+          }
+        }
+        tmem_store32(tmem + lane_base + kACol0 + (uint32_t)as * 32u, o);
+        tmem_store_wait();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&a_full[as]);
+        mbar_arrive(&empty[s]);
+      }
+
+      // ---------------------------------------------------------- segment end: epilogue
+      // Taken by the warpgroup that expanded the segment's last K-tile.
+      const bool seg_last = (w + 1 == w1) || ((w + 1) % T == 0);
+      if (!seg_last) continue;
+      const int64_t sg = w / T;  // segment = (token tile, row block)
+      const int64_t seg_begin = sg * T;
+      const int64_t mtile = sg / p.RB;
+      const int64_t rb = sg % p.RB;
+      const int64_t nrow = rb * kRows + r;
+      const float sc = (ES == 1 && nrow < p.N) ? p.scale[nrow] : 1.f;
+      if (!dead) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&d_full[grp], dph, p.timeout_ns));
+        if (!ok) {
+          dead = true;
+          set_status(p.status, kStatusTimeout);
+        }
+      }
+      dph ^= 1u;
+      tc_fence_after();
+      // this CTA ran the whole segment: its first and its last K-tile
+      const bool complete = seg_begin >= w0 && (w + 1) % T == 0;
+      const int my_slot = (sg == sg_first) ? 0 : 1;
+      const int64_t part = (int64_t)kRows * tp.ntok;  // floats per partial slot
+      float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * part;
+      for (int c0 = 0; c0 < tp.ntok; c0 += 32) {
+        uint32_t v[32];
+        if (!dead) {
+          tmem_load32(tmem + lane_base + (uint32_t)c0, v);
+          tmem_load_wait();
+        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          if (c0 + i >= tp.ntok) break;  // ntok is a multiple of 16, not always of 32
+          const int64_t tok = mtile * tp.ntok + c0 + i;
+          const float a = __uint_as_float(v[i]);
+          if (complete) {
+            if (tok < p.M && nrow < p.N) p.y[tok * p.N + nrow] = float_to_bf16_bits_rn(a * sc);
+          } else {
+            __stcg(wsp + (int64_t)(c0 + i) * kRows + r, a);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&d_empty[grp]);
+      if (!complete) {
+        const int bar = 1 + grp;
+        __threadfence();
+        named_bar_sync(bar, 128);
+        const int64_t i_first = owner_of(seg_begin, p.W, p.G);
+        const int64_t i_last = owner_of(seg_begin + T - 1, p.W, p.G);
+        const int sf = (range_begin(i_first, p.W, p.G) / T == sg) ? 0 : 1;
+        int* ctr = p.cnt + i_first * 2 + sf;
+        if (tid128 == 0) {
+          const int old = atomicAdd(ctr, 1);
+          s_flag[grp] = (old == (int)(i_last - i_first)) ? 1 : 0;
+        }
+        named_bar_sync(bar, 128);
+        if (s_flag[grp]) {
+          __threadfence();
+          // 32 tokens at a time: each contributor's 32 partials are independent loads
+          for (int c0 = 0; c0 < tp.ntok; c0 += 32) {
+            float sum[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) sum[i] = 0.f;
+            for (int64_t ci = i_first; ci <= i_last; ++ci) {
+              const int sl = (range_begin(ci, p.W, p.G) / T == sg) ? 0 : 1;
+              const float* src = p.ws + (ci * 2 + sl) * part + (int64_t)c0 * kRows + r;
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (c0 + i < tp.ntok) sum[i] += __ldcg(src + (int64_t)i * kRows);
+            }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int64_t tok = mtile * tp.ntok + c0 + i;
+              if (c0 + i < tp.ntok && tok < p.M && nrow < p.N)
+                p.y[tok * p.N + nrow] = float_to_bf16_bits_rn(sum[i] * sc);
+            }
+          }
+          if (tid128 == 0) atomicExch(ctr, 0);
+        }
+        named_bar_sync(bar, 128);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::mutex g_encode_mu;
+
+sp_status get_encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
+  std::lock_guard<std::mutex> lk(g_encode_mu);
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn) {
+      cudaGetLastError();
+      return SP_ERR_CUDA;
+    }
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  *out = g_encode;
+  return SP_OK;
+}
+
+int grid_tc(const sp_matrix* h, int64_t W) { return (int)std::min<int64_t>(h->num_sms, W); }
+
+int ntok_for(int64_t M) {
+  const int64_t n = std::min<int64_t>(kMaxNtok, (M + 15) / 16 * 16);
+  return (int)std::max<int64_t>(16, n);
+}
+
+template <int ES>
+sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, size_t smem, cudaStream_t stream) {
+  auto kern = linear_tc_kernel<ES>;
+  static bool configured[kMaxDevices] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
+  if (!configured[dev]) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemLimit) != cudaSuccess) {
+      cudaGetLastError();
+      return SP_ERR_CUDA;
+    }
+    configured[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)tp.p.G);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, kern, tp, map) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
+  return SP_OK;
+}
+
+}  // namespace
+
+size_t workspace_bytes_tc(const sp_matrix* h, int64_t M) {
+  const int ntok = ntok_for(M);
+  const int64_t mt = (M + ntok - 1) / ntok;
+  const int64_t W = mt * h->RB * h->T;
+  const size_t G = (size_t)grid_tc(h, W);
+  return ws_counter_bytes(h->num_sms) + 2 * G * kRows * (size_t)ntok * sizeof(float);
+}
+
+sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
+                           cudaStream_t stream) {
+  if (!ws || ws_bytes < workspace_bytes_tc(h, M)) return SP_ERR_WORKSPACE;
+  if (M > ((int64_t)1 << 31) / kMaxNtok) return SP_ERR_UNSUPPORTED;
+  PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  sp_status st = get_encoder(&encode);
+  if (st != SP_OK) return st;
+  TcParams tp{};
+  LinearParams& p = tp.p;
+  p.buf = h->d_buf;
+  p.off = h->d_off;
+  p.scale = h->d_scale;
+  p.x = x;
+  p.y = y;
+  p.status = device_status_ptr();
+  p.N = h->N;
+  p.K = h->K;
+  p.T = h->T;
+  p.RB = h->RB;
+  p.M = (int32_t)M;
+  tp.ntok = ntok_for(M);
+  tp.mt = (int32_t)((M + tp.ntok - 1) / tp.ntok);
+  p.W = (int64_t)tp.mt * h->RB * h->T;
+  p.G = grid_tc(h, p.W);
+  p.cnt = reinterpret_cast<int*>(ws);
+  p.ws = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms));
+  p.timeout_ns = wait_timeout_ns();
+  tp.b_bytes = (uint32_t)tp.ntok * 128u;
+  tp.chunk_off = (tp.b_bytes + 1023u) / 1024u * 1024u;
+  p.chunk_region = (uint32_t)((h->max_chunk + 1023) / 1024 * 1024);
+  p.slot_bytes = tp.chunk_off + p.chunk_region;
+  // base alignment + barriers (2 per slot, 2 per A stage, 2 for D), TMEM address, flag
+  const size_t tail = 1024 + 8 * (2 * kMaxSlots + 2 * kAStages + 2 * kExpGroups) + 4 + 4 * kExpGroups + 16;
+  const int slots = (int)std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes);
+  if (slots < 2) return SP_ERR_UNSUPPORTED;
+  p.slots = slots;
+  // at least 116 KB so that two CTAs never share an SM (each allocates 512 TMEM columns)
+  const size_t smem = std::max<size_t>((size_t)slots * p.slot_bytes + tail, 116 * 1024);
+
+  // x [M, K] bf16, box = 64 K-elements x ntok tokens, 128-byte swizzle; rows past M and
+  // columns past K read as zero.
+  CUtensorMap map;
+  const cuuint64_t gdim[2] = {(cuuint64_t)h->K, (cuuint64_t)M};
+  const cuuint64_t gstride[1] = {(cuuint64_t)h->K * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kTileK, (cuuint32_t)tp.ntok};
+  const cuuint32_t estride[2] = {1, 1};
+  if (encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(x), gdim, gstride, box, estride,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return SP_ERR_CUDA;
+  return h->esize == 2 ? launch_tc_es<2>(tp, map, smem, stream) : launch_tc_es<1>(tp, map, smem, stream);
+}
+
+}  // namespace sp

@@ -10,7 +10,7 @@ from tests import gpu_util as gu
 
 pytestmark = pytest.mark.gpu
 
-PATHS = ["cuda_core"]
+PATHS = ["cuda_core", "tensor_core"]
 
 
 @pytest.fixture(scope="module")
