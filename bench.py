@@ -44,6 +44,8 @@ def parse():
     ap.add_argument("--path", default="auto", choices=["auto", "cuda_core", "tensor_core"])
     ap.add_argument("--sweep", default="1,4,16", help="extra batch sizes reported under per_m ('' = none)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle leg")
+    ap.add_argument("--no-stack", action="store_true", help="skip the INT8 32-layer stack section")
+    ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--single", default="", choices=["", *SHAPES],
                     help="profiling aid: time one layer-0 linear of this shape (--warmup then --steps launches)")
     return ap.parse_args()
@@ -78,6 +80,103 @@ def load_peaks():
             d = json.load(f)
         return float(d["hbm_gbs"]), "measured"
     return 6800.0, "fallback"
+
+
+def load_tensor_peak():
+    """bf16 dense tensor peak (TFLOP/s) for a kernel timed alone (burst figure)."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    return 1900.0, "fallback"
+
+
+def time_graph(g, steps, warmup):
+    import torch
+
+    for _ in range(warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        g.replay()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / steps
+
+
+def stack_section(args, peak_gbs):
+    """configs[4]: 32-layer linear stack, 70% INT8 weights with fp32 per-row scales,
+    layers chained by residual adds, one CUDA graph per decode step."""
+    import numpy as np
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+    from paper_2405_03594_gb300.stack import LinearStack
+
+    st = LinearStack(layers=LAYERS, pct=args.pct, int8=True, max_m=64)
+    out = {"workload": f"llama2-7b linear stack, {LAYERS} layers, {args.pct}% INT8 weights + fp32 per-row scales, "
+                       "residual chain, one CUDA graph per step",
+           "weight_bytes": st.weight_bytes(), "per_m": {}}
+    for M in (1, 16, 64):
+        x = synth.activations(M, 4096, synth.rng(0, 0, 0, synth.STREAM_X))
+        st.set_input(torch.from_numpy(x.view(np.int16)).to(st.dev).view(torch.bfloat16))
+        g = st.capture(M)
+        steps = max(3, min(args.steps, 100))
+        ms = time_graph(g, steps, max(3, args.warmup))
+        sp.check()
+        finite = bool(torch.isfinite(st.h[:M].float()).all().item())
+        bytes_step = st.weight_bytes() + LAYERS * 2 * M * (4096 * 4 + 12288 + 22016 + 11008)
+        out["per_m"][str(M)] = {"tok_s": M / (ms * 1e-3), "ms_per_step": ms, "gbs": bytes_step / (ms * 1e-3) / 1e9,
+                                "frac_of_peak": bytes_step / (ms * 1e-3) / 1e9 / peak_gbs,
+                                "launches_per_step": st.launches_per_step(M), "activations_finite": finite}
+        del g
+    del st
+    torch.cuda.empty_cache()
+    return out
+
+
+def prefill_section(args):
+    """configs[2]: the four shapes at 50% and 70%, x [2048, K], tensor-core path."""
+    import numpy as np
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+
+    peak, kind = load_tensor_peak()
+    dev = torch.device("cuda", 0)
+    M = 2048
+    res = {"M": M, "peak_tflops": peak, "peak_kind": f"of {kind} (bf16_tflops, burst)", "shapes": {}}
+    for pct in (50, 70):
+        for name in SHAPES:
+            W, mask, _ = synth.layer_inputs(name, pct, 1, seed=0, layer=0)
+            N, K = W.shape
+            x = synth.activations(M, K, synth.rng(0, 0, synth.PROJ_IDS[name], synth.STREAM_X))
+            h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
+                            torch.from_numpy(mask).to(dev))
+            xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+            y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+            ws = torch.zeros(max(h.workspace_size(M), 256), dtype=torch.uint8, device=dev)
+            for _ in range(3):
+                h.linear(xd, out=y, workspace=ws, path="tensor_core")
+            torch.cuda.synchronize()
+            reps = 10
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(reps):
+                h.linear(xd, out=y, workspace=ws, path="tensor_core")
+            b.record()
+            torch.cuda.synchronize()
+            sp.check()
+            us = a.elapsed_time(b) / reps * 1e3
+            nz = 2.0 * M * int(h.info.nnz) / (us * 1e-6) / 1e12
+            dense = 2.0 * M * N * K / (us * 1e-6) / 1e12
+            res["shapes"][f"{name}@{pct}%"] = {"us": us, "tflops_nonzero": nz, "frac_nonzero": nz / peak,
+                                               "tflops_dense_executed": dense, "frac_dense_executed": dense / peak}
+            del h, xd, y, ws
+    torch.cuda.empty_cache()
+    return res
 
 
 def kernel_source_hash():
@@ -393,6 +492,12 @@ def run_ours(args):
             fro = max(fro, float(np.linalg.norm(y - ref) / np.linalg.norm(ref)))
         parity = {"max_err_over_max_ref": worst, "rel_fro": fro, "ok": worst <= 1e-2 and fro <= 5e-3}
 
+    # ---------------------------------------------------------------- configs[4] and configs[2]
+    del mats
+    torch.cuda.empty_cache()
+    stack = None if args.no_stack else stack_section(args, peak_gbs)
+    prefill = None if (args.no_prefill or world > 1) else prefill_section(args)
+
     if rank == 0:
         launches_per_step = LAYERS * len(SHAPES) * ((M + 15) // 16)
         line = {
@@ -417,6 +522,8 @@ def run_ours(args):
             "clocks": clocks,
             "step_gbs": r["step_gbs"],
             "parity_layer0": parity,
+            "stack_int8": stack,
+            "prefill": prefill,
             "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
                                "frac_of_peak": v["step_gbs"] / peak_gbs,
                                "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),

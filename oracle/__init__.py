@@ -50,6 +50,8 @@ def _bind(lib):
     lib.or_linear_int8.argtypes = [P, I64, P, P, P, I64, I64, P]
     lib.or_linear_from_format.argtypes = [P, P, I64, I64, ctypes.c_int, P, P, I64, P]
     lib.or_linear_from_format.restype = ctypes.c_int
+    lib.or_residual_add.argtypes = [P, P, P, I64, I64, P]
+    lib.or_mul_halves.argtypes = [P, I64, I64, P]
     lib.or_block_encode.argtypes = [P, ctypes.c_int, P, P]
     lib.or_block_encode.restype = ctypes.c_int
     return lib
@@ -158,3 +160,23 @@ def block_encode(elems) -> tuple[list[int], int]:
     m = np.zeros(1, dtype=np.uint64)
     c = _load().or_block_encode(_p(e), int(e.size), _p(vals), _p(m))
     return [int(v) for v in vals[:c]], int(m[0])
+
+
+def residual_add(h: np.ndarray, a: np.ndarray, r: np.ndarray) -> np.ndarray:
+    """float64 h + a + r (bf16 inputs, r broadcast over rows), before rounding."""
+    h = np.ascontiguousarray(h, dtype=np.uint16)
+    a = np.ascontiguousarray(a, dtype=np.uint16)
+    r = np.ascontiguousarray(r, dtype=np.uint16)
+    M, N = h.shape
+    out = np.zeros((M, N), dtype=np.float64)
+    _load().or_residual_add(_p(h), _p(a), _p(r), M, N, _p(out))
+    return out
+
+
+def mul_halves(g: np.ndarray) -> np.ndarray:
+    """float64 g[:, :F] * g[:, F:] (bf16 input), before rounding."""
+    g = np.ascontiguousarray(g, dtype=np.uint16)
+    M, F2 = g.shape
+    out = np.zeros((M, F2 // 2), dtype=np.float64)
+    _load().or_mul_halves(_p(g), M, F2 // 2, _p(out))
+    return out

@@ -245,3 +245,18 @@ int or_block_encode(const int16_t* elems, int n, int16_t* values, uint64_t* mask
   *mask = m;
   return c;
 }
+
+/* Glue of the linear-stack decode step (not part of the paper's method: the benchmark
+ * chains the linears of each block with residual adds, no attention or normalisation).
+ * Results in float64, before any rounding. */
+void or_residual_add(const uint16_t* h, const uint16_t* a, const uint16_t* r, int64_t M, int64_t N, double* out) {
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t j = 0; j < N; ++j)
+      out[m * N + j] = or_bf16_to_double(h[m * N + j]) + or_bf16_to_double(a[m * N + j]) + or_bf16_to_double(r[j]);
+}
+
+void or_mul_halves(const uint16_t* g, int64_t M, int64_t F, double* out) {
+  for (int64_t m = 0; m < M; ++m)
+    for (int64_t j = 0; j < F; ++j)
+      out[m * F + j] = or_bf16_to_double(g[m * 2 * F + j]) * or_bf16_to_double(g[m * 2 * F + F + j]);
+}

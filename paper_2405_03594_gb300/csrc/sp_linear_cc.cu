@@ -63,11 +63,41 @@ __device__ __forceinline__ uint16_t i8_to_bf16(uint32_t byte) {
   return (uint16_t)(__float_as_uint(f) >> 16);
 }
 
-template <int ES>
-__device__ __forceinline__ uint16_t load_w(const uint8_t* vals, int idx) {
-  if (ES == 2) return reinterpret_cast<const uint16_t*>(vals)[idx];
-  return i8_to_bf16(vals[idx]);
+__device__ __forceinline__ uint32_t lds32(uint32_t saddr) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(saddr));
+  return v;
 }
+// Low 32 bits of ({hi, lo} >> n), n clamped to 32.
+__device__ __forceinline__ uint32_t funnel_r(uint32_t lo, uint32_t hi, uint32_t n) {
+  uint32_t r;
+  asm("shf.r.clamp.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(lo), "r"(hi), "r"(n));
+  return r;
+}
+// Clear bit j (no-op for j = -1).
+__device__ __forceinline__ uint32_t clear_bit(uint32_t v, int j) { return v & ~bit32(j); }
+
+// One chain's value stream, walked from its highest-column value downward.  The values
+// are bf16 halves at byte address `top` (the highest) and below; every second step
+// loads one aligned 32-bit word, and a funnel shift realigns odd starting positions.
+struct Stream16 {
+  uint32_t addr;   // byte address of the aligned word holding the next pair's first value
+  uint32_t cur;    // that word
+  uint32_t shift;  // 16 if the stream starts at a low half (even index), else 32
+  __device__ __forceinline__ void init(uint32_t top_byte) {
+    addr = top_byte & ~3u;
+    cur = lds32(addr);
+    shift = (top_byte & 2u) ? 32u : 16u;
+  }
+  // next two values: first in the high half, second in the low half
+  __device__ __forceinline__ uint32_t next_pair() {
+    addr -= 4;
+    const uint32_t below = lds32(addr);
+    const uint32_t w = funnel_r(below, cur, shift);
+    cur = below;
+    return w;
+  }
+};
 
 template <int M, int ES>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const LinearParams p) {
@@ -199,28 +229,76 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
       const int top_lo = e0 + plo - 1;  // highest-column value of the low half
       const int top_hi = e0 + pc - 1;   // ... of the high half
       const int iters = (int)__reduce_max_sync(0xffffffffu, (unsigned)max(plo, pc - plo));
-#pragma unroll 2
-      for (int q = 0; q < iters; ++q) {
-        const int jl = msb32(lo), jh = msb32(hi);
-        lo &= ~bit32(jl);
-        hi &= ~bit32(jh);
-        const bool al = jl >= 0, ah = jh >= 0;
-        uint16_t wl = 0, wh = 0;
-        if (al) wl = load_w<ES>(vals, top_lo - q);
-        if (ah) wh = load_w<ES>(vals, top_hi - q);
+      float accl[M <= 4 ? M : 1], acch[M <= 4 ? M : 1];
 #pragma unroll
-        for (int r = 0; r < MP; ++r) {
-          const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
-          const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
-          if (al) {
-            acc[2 * r] = fma_bf16(wl, lo16(xl), acc[2 * r]);
-            if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wl, hi16(xl), acc[2 * r + 1]);
-          }
-          if (ah) {
-            acc[2 * r] = fma_bf16(wh, lo16(xh), acc[2 * r]);
-            if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wh, hi16(xh), acc[2 * r + 1]);
+      for (int m = 0; m < (M <= 4 ? M : 1); ++m) {
+        accl[m] = 0.f;
+        acch[m] = 0.f;
+      }
+      if (ES == 2 && M <= 4) {
+        // bf16, small batch: two chain steps per loop trip share one word load per chain,
+        // and each chain keeps its own accumulators
+        Stream16 sl, sh;
+        const uint32_t vbase = smem_u32(vals);
+        sl.init(vbase + 2u * (uint32_t)top_lo);
+        sh.init(vbase + 2u * (uint32_t)top_hi);
+        for (int q = 0; q < iters; q += 2) {
+          const uint32_t wl = sl.next_pair(), wh = sh.next_pair();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int jl = msb32(lo), jh = msb32(hi);
+            lo = clear_bit(lo, jl);
+            hi = clear_bit(hi, jh);
+            const uint16_t vl = h == 0 ? hi16(wl) : lo16(wl);
+            const uint16_t vh = h == 0 ? hi16(wh) : lo16(wh);
+#pragma unroll
+            for (int r = 0; r < MP; ++r) {
+              const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+              const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+              if (jl >= 0) {
+                accl[2 * r] = fma_bf16(vl, lo16(xl), accl[2 * r]);
+                if (2 * r + 1 < M) accl[2 * r + 1] = fma_bf16(vl, hi16(xl), accl[2 * r + 1]);
+              }
+              if (jh >= 0) {
+                acch[2 * r] = fma_bf16(vh, lo16(xh), acch[2 * r]);
+                if (2 * r + 1 < M) acch[2 * r + 1] = fma_bf16(vh, hi16(xh), acch[2 * r + 1]);
+              }
+            }
           }
         }
+      } else {
+        // larger batches (or int8 values): one value per chain step, one accumulator set
+#pragma unroll 2
+        for (int q = 0; q < iters; ++q) {
+          const int jl = msb32(lo), jh = msb32(hi);
+          lo = clear_bit(lo, jl);
+          hi = clear_bit(hi, jh);
+          uint16_t wl = 0, wh = 0;
+          if (ES == 2) {
+            if (jl >= 0) wl = reinterpret_cast<const uint16_t*>(vals)[top_lo - q];
+            if (jh >= 0) wh = reinterpret_cast<const uint16_t*>(vals)[top_hi - q];
+          } else {
+            if (jl >= 0) wl = i8_to_bf16(vals[top_lo - q]);
+            if (jh >= 0) wh = i8_to_bf16(vals[top_hi - q]);
+          }
+#pragma unroll
+          for (int r = 0; r < MP; ++r) {
+            const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+            const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+            if (jl >= 0) {
+              acc[2 * r] = fma_bf16(wl, lo16(xl), acc[2 * r]);
+              if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wl, hi16(xl), acc[2 * r + 1]);
+            }
+            if (jh >= 0) {
+              acc[2 * r] = fma_bf16(wh, lo16(xh), acc[2 * r]);
+              if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wh, hi16(xh), acc[2 * r + 1]);
+            }
+          }
+        }
+      }
+      if (ES == 2 && M <= 4) {
+#pragma unroll
+        for (int m = 0; m < (M <= 4 ? M : 1); ++m) acc[m] += accl[m] + acch[m];
       }
     }
     __syncwarp();

@@ -23,9 +23,10 @@ STATUS = {
     0: "SP_OK", 1: "SP_ERR_INVALID_ARG", 2: "SP_ERR_UNSUPPORTED", 3: "SP_ERR_ALIGNMENT", 4: "SP_ERR_CUDA",
     5: "SP_ERR_OUT_OF_MEMORY", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_BAD_HANDLE", 8: "SP_ERR_WORKSPACE",
 }
-# every function declared in include/sp.h
+# every function declared in include/sp.h and include/sp_stack.h
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_linear_noalloc",
-           "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string"]
+           "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
+           "sp_copy_columns", "sp_residual_add", "sp_mul_halves"]
 
 
 class SpError(RuntimeError):
@@ -61,6 +62,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_info.argtypes = [P, ctypes.POINTER(SpInfo)]
     lib.sp_copy_out.argtypes = [P, P, SZ, P, SZ]
     lib.sp_check.argtypes = [P]
+    lib.sp_copy_columns.argtypes = [P, P, I64, I64, I64, I64, P]
+    lib.sp_residual_add.argtypes = [P, P, P, I64, I64, P]
+    lib.sp_mul_halves.argtypes = [P, P, I64, I64, P]
     lib.sp_status_string.argtypes = [ctypes.c_int]
     lib.sp_status_string.restype = ctypes.c_char_p
     for name in EXPORTS:
@@ -214,6 +218,27 @@ def workspace_for(nbytes: int, device) -> torch.Tensor:
         ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=torch.device("cuda", key))
         _ws_cache[key] = ws
     return ws
+
+
+def copy_columns(out: torch.Tensor, inp: torch.Tensor, col0: int, stream=None) -> torch.Tensor:
+    """out[m, :] = inp[m, col0 : col0 + out.shape[1]] (bf16, in a libsp kernel)."""
+    M, n = out.shape
+    _check(_lib.sp_copy_columns(_ptr(out), _ptr(inp), M, inp.shape[1], col0, n, _stream(stream)), "sp_copy_columns")
+    return out
+
+
+def residual_add(h: torch.Tensor, a: torch.Tensor, r: torch.Tensor, stream=None) -> torch.Tensor:
+    """h = bf16(h + a + r) in place, r broadcast over rows."""
+    M, N = h.shape
+    _check(_lib.sp_residual_add(_ptr(h), _ptr(a), _ptr(r), M, N, _stream(stream)), "sp_residual_add")
+    return h
+
+
+def mul_halves(out: torch.Tensor, g: torch.Tensor, stream=None) -> torch.Tensor:
+    """out = bf16(g[:, :F] * g[:, F:]) with F = out.shape[1]."""
+    M, F = out.shape
+    _check(_lib.sp_mul_halves(_ptr(out), _ptr(g), M, F, _stream(stream)), "sp_mul_halves")
+    return out
 
 
 def check(stream=None):

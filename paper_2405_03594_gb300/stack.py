@@ -1,0 +1,132 @@
+"""Decode step of a Llama-2-7B linear-only stack on libsp.
+
+Per layer, four fused sparse linears and the elementwise glue of include/sp_stack.h:
+
+    qkv = x.Wqkv^T            [M, 12288]      (sparse linear)
+    v   = qkv[:, 8192:12288]                   (sp_copy_columns)
+    h   = h + v.Wo^T + r_l                      (sparse linear, sp_residual_add)
+    gu  = h.Wgu^T             [M, 22016]      (sparse linear)
+    a   = gu[:, :11008] * gu[:, 11008:]        (sp_mul_halves)
+    h   = h + a.Wdown^T + r'_l                  (sparse linear, sp_residual_add)
+
+All arithmetic runs in libsp kernels; PyTorch only holds the buffers.  The layers are
+device copies of one seeded layer (each its own HBM buffers), so a step streams the
+full 32-layer weight set.  `capture()` records one step as a single CUDA graph.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import sp, synth
+
+SHAPES = ("qkv", "o", "gate_up", "down")
+D_MODEL = 4096
+D_FF = 11008
+# Initial weight scale of the stack: with N(0, 0.02^2) weights, 70% magnitude masks and
+# no normalisation, the gate*up product makes activations overflow within a few layers;
+# N(0, 0.004^2) keeps them O(10) through 32 layers.
+STACK_WEIGHT_STD = 0.004
+
+
+def host_layer(pct: int, int8: bool, seed: int = 0, std: float = STACK_WEIGHT_STD):
+    """Seeded host inputs of one layer: {shape: (values, mask, scale or None)}."""
+    out = {}
+    for name in SHAPES:
+        N, K = synth.LLAMA2_7B_SHAPES[name]
+        p = synth.PROJ_IDS[name]
+        W = synth.weight(N, K, synth.rng(seed, 0, p, synth.STREAM_W), std=std)
+        mask = synth.magnitude_mask(W, pct)
+        if int8:
+            q, s = synth.quantize_int8(W, mask)
+            out[name] = (q, mask, s)
+        else:
+            out[name] = (W, mask, None)
+    return out
+
+
+class LinearStack:
+    def __init__(self, layers: int = 32, pct: int = 70, int8: bool = True, max_m: int = 64, seed: int = 0,
+                 device=None, host=None, path: str = "auto"):
+        self.dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+        self.layers, self.max_m, self.path = layers, max_m, path
+        self.host = host_layer(pct, int8, seed) if host is None else host
+        self.mats = {}
+        for name in SHAPES:
+            vals, mask, s = self.host[name]
+            if s is not None:
+                h0 = sp.compress(torch.from_numpy(vals).to(self.dev), torch.from_numpy(mask).to(self.dev),
+                                 torch.from_numpy(s).to(self.dev))
+            else:
+                h0 = sp.compress(torch.from_numpy(vals.view(np.int16)).to(self.dev).view(torch.bfloat16),
+                                 torch.from_numpy(mask).to(self.dev))
+            self.mats[name] = [h0] + [h0.clone() for _ in range(layers - 1)]
+        g = synth.rng(seed, 0, 9, synth.STREAM_RESID)
+        r = synth.activations(2 * layers, D_MODEL, g)
+        rt = torch.from_numpy(r.view(np.int16)).to(self.dev).view(torch.bfloat16)
+        self.r1 = [rt[2 * l].contiguous() for l in range(layers)]
+        self.r2 = [rt[2 * l + 1].contiguous() for l in range(layers)]
+        bf = dict(dtype=torch.bfloat16, device=self.dev)
+        self.h = torch.zeros((max_m, D_MODEL), **bf)
+        self.x0 = torch.zeros((max_m, D_MODEL), **bf)  # the step's input token embeddings
+        self.qkv = torch.empty((max_m, 3 * D_MODEL), **bf)
+        self.v = torch.empty((max_m, D_MODEL), **bf)
+        self.o = torch.empty((max_m, D_MODEL), **bf)
+        self.gu = torch.empty((max_m, 2 * D_FF), **bf)
+        self.a = torch.empty((max_m, D_FF), **bf)
+        self.d = torch.empty((max_m, D_MODEL), **bf)
+        ws = max(self.mats[n][0].workspace_size(max_m) for n in SHAPES)
+        self.ws = torch.zeros(max(ws, 256), dtype=torch.uint8, device=self.dev)
+        torch.cuda.synchronize()
+
+    def weight_bytes(self) -> int:
+        return self.layers * sum(int(self.mats[n][0].info.bytes) + int(self.mats[n][0].info.scale_bytes)
+                                 for n in SHAPES)
+
+    def launches_per_step(self, M: int, reset: bool = True) -> int:
+        """libsp kernels per step: four sparse linears and four glue kernels per layer
+        (the CUDA-core family takes at most 16 batch rows per launch), plus the input copy."""
+        per_linear = (M + 15) // 16 if self.path == "cuda_core" else 1
+        return self.layers * (4 * per_linear + 4) + (1 if reset else 0)
+
+    def set_input(self, x: torch.Tensor):
+        """Token embeddings [M, 4096] bf16 for the next steps."""
+        M = x.shape[0]
+        self.x0[:M].copy_(x)
+        self.h[:M].copy_(x)
+
+    def step(self, M: int, record=None, stream=None, reset: bool = False):
+        """One decode step for the first M rows of self.h (in place); with reset=True it
+        starts from the saved input (set_input).  If `record` is a list, each linear's
+        (layer, shape, input, output) copies are appended to it."""
+        kw = dict(workspace=self.ws, path=self.path, stream=stream)
+        h, qkv, v, o, gu, a, d = (t[:M] for t in (self.h, self.qkv, self.v, self.o, self.gu, self.a, self.d))
+        if reset:
+            sp.copy_columns(h, self.x0[:M], 0, stream=stream)
+        for l in range(self.layers):
+            self.mats["qkv"][l].linear(h, out=qkv, **kw)
+            if record is not None:
+                record.append((l, "qkv", h.clone(), qkv.clone()))
+            sp.copy_columns(v, qkv, 2 * D_MODEL, stream=stream)
+            self.mats["o"][l].linear(v, out=o, **kw)
+            if record is not None:
+                record.append((l, "o", v.clone(), o.clone()))
+            sp.residual_add(h, o, self.r1[l], stream=stream)
+            self.mats["gate_up"][l].linear(h, out=gu, **kw)
+            if record is not None:
+                record.append((l, "gate_up", h.clone(), gu.clone()))
+            sp.mul_halves(a, gu, stream=stream)
+            self.mats["down"][l].linear(a, out=d, **kw)
+            if record is not None:
+                record.append((l, "down", a.clone(), d.clone()))
+            sp.residual_add(h, d, self.r2[l], stream=stream)
+
+    def capture(self, M: int) -> torch.cuda.CUDAGraph:
+        """One decode step from the saved input, recorded as a single CUDA graph."""
+        self.step(M, reset=True)  # warm: per-device kernel attributes are set outside the capture
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step(M, reset=True)
+        torch.cuda.synchronize()
+        return g

@@ -8,7 +8,8 @@ import re
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADER = os.path.join(ROOT, "include", "sp.h")
+HEADERS = [os.path.join(ROOT, "include", h) for h in sorted(os.listdir(os.path.join(ROOT, "include")))
+           if h.endswith(".h")]
 
 
 @pytest.fixture(scope="module")
@@ -23,15 +24,28 @@ def lib():
 
 
 def declared_functions():
-    src = open(HEADER).read()
-    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:sp_status|const char\s*\*)\s+(sp_\w+)\s*\(", src, flags=re.M)))
+    names = set()
+    for hdr in HEADERS:
+        src = re.sub(r"/\*.*?\*/", "", open(hdr).read(), flags=re.S)
+        names |= set(re.findall(r"^\s*(?:sp_status|const char\s*\*)\s+(sp_\w+)\s*\(", src, flags=re.M))
+    return sorted(names)
 
 
 def test_header_declares_the_boundary():
     names = declared_functions()
-    for n in ["sp_compress", "sp_decompress", "sp_linear", "sp_free", "sp_workspace_size", "sp_check"]:
+    for n in ["sp_compress", "sp_decompress", "sp_linear", "sp_free", "sp_workspace_size", "sp_check",
+              "sp_residual_add", "sp_mul_halves", "sp_copy_columns"]:
         assert n in names
+
+
+def test_glue_argument_checks(lib):
+    P = ctypes.c_void_p
+    f = P(1 << 20)
+    assert lib.sp_residual_add(None, f, f, 2, 8, None) == 1
+    assert lib.sp_residual_add(f, f, f, 2, 12, None) == 2
+    assert lib.sp_residual_add(P((1 << 20) + 4), f, f, 2, 8, None) == 3
+    assert lib.sp_mul_halves(f, f, 2, 0, None) == 0  # empty: nothing to launch
+    assert lib.sp_copy_columns(f, f, 2, 16, 8, 16, None) == 1  # in_stride < col0 + ncols
 
 
 def test_every_declared_symbol_is_exported(lib):
