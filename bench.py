@@ -39,7 +39,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--m", type=int, default=16, help="decode batch (tokens per step)")
+    ap.add_argument("--m", type=int, default=1, help="decode batch (tokens per step)")
     ap.add_argument("--pct", type=int, default=70)
     ap.add_argument("--path", default="auto", choices=["auto", "cuda_core", "tensor_core"])
     ap.add_argument("--sweep", default="1,4,16", help="extra batch sizes reported under per_m ('' = none)")

@@ -130,9 +130,9 @@ sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y
  * input and output buffers from a host framework or plugin interface that owns all
  * device memory, and some run latency-critical loops where cudaMalloc/cudaFree would
  * synchronise the device: neither can supply sp_linear's workspace.  This call runs the
- * same CUDA-core decode kernel with the same launch configuration, using instead a
- * scratch array of 16 MiB that the library keeps on every GPU that loads it (held until
- * the process exits).  It calls no cudaMalloc, cudaFree or other allocating routine.
+ * CUDA-core decode kernel in its stream-K configuration, using instead a scratch array
+ * of 16 MiB that the library keeps on every GPU that loads it (held until the process
+ * exits).  It calls no cudaMalloc, cudaFree or other allocating routine.
  *   x_dev [m, K] bf16, y_dev [m, N] bf16, as for sp_linear.
  *   Returns SP_ERR_WORKSPACE if the kernel would need more scratch than the array holds.
  *   The first call on a device looks up the array's device address (set-up, once per

@@ -117,6 +117,9 @@ sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y
     return SP_ERR_CUDA;
   }
   if (dev != h->device) return SP_ERR_INVALID_ARG;
+  // The documented contract, whatever kernel runs: a workspace of sp_workspace_size bytes.
+  if (!workspace_dev || workspace_bytes < std::max(workspace_bytes_cc(h, m), workspace_bytes_tc(h, m)))
+    return SP_ERR_WORKSPACE;
   if (path == SP_PATH_TENSOR_CORE || (path == SP_PATH_AUTO && m > kCudaCoreMaxM))
     return launch_linear_tc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
                             workspace_bytes, (cudaStream_t)stream);

@@ -64,6 +64,9 @@ struct LinearParams {
   uint32_t slot_bytes;  // bytes per ring slot (chunk region + x tile region)
   uint32_t chunk_region;// bytes reserved for the chunk inside a slot
   uint64_t timeout_ns;
+  int32_t cluster;      // CUDA-core kernel: > 1 = split each row block over this many CTAs of
+                        // one thread-block cluster; <= 1 = stream-K over the workspace
+  uint32_t part_off;    // cluster mode: shared-memory offset of the CTA's FP32 partial
 };
 
 // Workspace layout, fixed per device so that calls with different grids can share it:
@@ -142,11 +145,57 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// A warp-wide window of 32 consecutive chunk offsets held one per lane, so that a
+// producer needs one coalesced global load per 31 chunks instead of a dependent L2
+// round trip per chunk.  Every lane of the warp must call at() with the same c.
+struct OffsetWindow {
+  const uint64_t* off;
+  int64_t n_off;  // entries in off[]
+  int64_t base;
+  uint64_t v;
+  __device__ __forceinline__ void refill(int64_t c) {
+    base = c;
+    const int lane = threadIdx.x & 31;
+    v = (c + lane < n_off) ? __ldg(off + c + lane) : 0ull;
+  }
+  __device__ __forceinline__ void init(const uint64_t* o, int64_t n, int64_t c) {
+    off = o;
+    n_off = n;
+    refill(c);
+  }
+  // (off[c], off[c + 1])
+  __device__ __forceinline__ void at(int64_t c, uint64_t* o0, uint64_t* o1) {
+    if (c < base || c + 1 - base >= 32) refill(c);
+    *o0 = __shfl_sync(0xffffffffu, v, (int)(c - base));
+    *o1 = __shfl_sync(0xffffffffu, v, (int)(c + 1 - base));
+  }
+};
+
 // Programmatic dependent launch: wait for the preceding grid in the stream (and its
 // memory) / allow the next grid to start its prologue.  No-ops without the launch
 // attribute.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+// Thread-block cluster helpers (every thread of every CTA of the cluster must take part).
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cta address -> the same offset in CTA `rank` of the cluster (shared::cluster window)
+__device__ __forceinline__ uint32_t cluster_map(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_cluster_f32(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
@@ -163,8 +212,10 @@ __device__ __forceinline__ uint16_t float_to_bf16_bits_rn(float f) {
 sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t K, sp_dtype dt, const float* scale,
                           sp_alloc_fn alloc, sp_free_fn free_fn, void* ctx, cudaStream_t stream, sp_matrix** out);
 sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream);
+// allow_cluster: split small row-block counts over thread-block clusters (no workspace
+// needed); otherwise stream-K with split-K partials in the workspace.
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool allow_cluster = true);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
 sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream);

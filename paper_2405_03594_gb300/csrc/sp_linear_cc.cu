@@ -99,17 +99,28 @@ struct Stream16 {
   }
 };
 
-template <int M, int ES>
+template <int M, int ES, bool CL>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
   uint64_t* empty = full + p.slots;
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
-  const int64_t w0 = range_begin(blockIdx.x, p.W, p.G);
-  const int64_t w1 = range_begin(blockIdx.x + 1, p.W, p.G);
   const int T = p.T;
   const int slots = p.slots;
+  constexpr bool clustered = CL;  // split-K over a thread-block cluster (else stream-K)
+  int64_t w0, w1;
+  uint32_t crank = 0;
+  if (clustered) {
+    // cluster c owns row block c; its CTA of rank r takes K-tiles [r*T/S, (r+1)*T/S)
+    const int64_t seg = blockIdx.x / p.cluster;
+    crank = cluster_rank();
+    w0 = seg * T + (int64_t)crank * T / p.cluster;
+    w1 = seg * T + (int64_t)(crank + 1) * T / p.cluster;
+  } else {
+    w0 = range_begin(blockIdx.x, p.W, p.G);
+    w1 = range_begin(blockIdx.x + 1, p.W, p.G);
+  }
 
   if (tid == 0) {
     for (int s = 0; s < slots; ++s) {
@@ -122,51 +133,63 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
 
   if (warp == kConsumerWarps) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      // Weight bytes do not depend on the previous kernel in the stream: the first
-      // ring fill is issued before griddepcontrol.wait; every x copy comes after it.
-      const uint64_t pol = policy_evict_first();
-      const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
-      {
-        int t = (int)(w0 % T);
-        for (int64_t i = 0; i < n_pre; ++i) {
-          const int64_t w = w0 + i;
-          const uint64_t o0 = p.off[w];
-          const uint32_t bytes = (uint32_t)(p.off[w + 1] - o0);
+    // The whole warp walks the chunk list (it shares the offset window); lane 0 issues.
+    // Weight bytes do not depend on the previous kernel in the stream: the first ring
+    // fill is issued before griddepcontrol.wait; every x copy comes after it.
+    const uint64_t pol = policy_evict_first();
+    OffsetWindow ow;
+    ow.init(p.off, p.W + 1, w0);
+    const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
+    {
+      int t = (int)(w0 % T);
+      for (int64_t i = 0; i < n_pre; ++i) {
+        uint64_t o0, o1;
+        ow.at(w0 + i, &o0, &o1);
+        if (lane == 0) {
+          const uint32_t bytes = (uint32_t)(o1 - o0);
           const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
           mbar_arrive_expect_tx(&full[i], bytes + (uint32_t)M * (uint32_t)valid * 2u);
           bulk_g2s_hint(smem + (size_t)i * p.slot_bytes, p.buf + o0, bytes, &full[i], pol);
-          if (++t == T) t = 0;
         }
+        if (++t == T) t = 0;
       }
-      pdl_wait();
-      pdl_launch_dependents();
-      int s = 0;
-      uint32_t ph = 0;
-      int t = (int)(w0 % T);
-      int64_t n_issued = 0;
-      for (int64_t w = w0; w < w1; ++w, ++n_issued) {
-        const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
-        const uint32_t xb = (uint32_t)valid * 2u;
-        uint8_t* slot = smem + (size_t)s * p.slot_bytes;
-        if (n_issued >= n_pre) {
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    int s = 0;
+    uint32_t ph = 0;
+    int t = (int)(w0 % T);
+    int64_t n_issued = 0;
+    bool failed = false;
+    for (int64_t w = w0; w < w1 && !failed; ++w, ++n_issued) {
+      const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
+      const uint32_t xb = (uint32_t)valid * 2u;
+      uint8_t* slot = smem + (size_t)s * p.slot_bytes;
+      if (n_issued >= n_pre) {
+        uint64_t o0, o1;
+        ow.at(w, &o0, &o1);
+        if (lane == 0) {
           if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
             set_status(p.status, kStatusTimeout);
-            break;
+            failed = true;
+          } else {
+            const uint32_t bytes = (uint32_t)(o1 - o0);
+            mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
+            bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
           }
-          const uint64_t o0 = p.off[w];
-          const uint32_t bytes = (uint32_t)(p.off[w + 1] - o0);
-          mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
-          bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
         }
+        failed = __shfl_sync(0xffffffffu, failed, 0);
+        if (failed) break;
+      }
+      if (lane == 0) {
 #pragma unroll
         for (int m = 0; m < M; ++m)
           bulk_g2s(slot + p.chunk_region + m * 128, p.x + (int64_t)m * p.K + (int64_t)kTileK * t, xb, &full[s]);
-        if (++t == T) t = 0;
-        if (++s == slots) {
-          s = 0;
-          ph ^= 1u;
-        }
+      }
+      if (++t == T) t = 0;
+      if (++s == slots) {
+        s = 0;
+        ph ^= 1u;
       }
     }
     return;
@@ -319,6 +342,35 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
     const int64_t seg_begin = rb_cur * T;
     const int64_t n = rb_cur * kRows + tid;
     const float sc = (ES == 1 && n < p.N) ? p.scale[n] : 1.f;
+    if constexpr (clustered) {
+      // Each CTA leaves its FP32 partial in its own shared memory; after a cluster barrier
+      // rank 0 adds the other ranks' partials in rank order (distributed shared memory)
+      // and writes y; a second barrier keeps every partial alive until then.
+      float* part = reinterpret_cast<float*>(smem + p.part_off);
+#pragma unroll
+      for (int m = 0; m < M; ++m) part[m * kRows + tid] = acc[m];
+      cluster_sync_all();
+      if (crank == 0) {
+        float sum[M];
+#pragma unroll
+        for (int m = 0; m < M; ++m) sum[m] = acc[m];
+        const uint32_t base = smem_u32(part) + 4u * (uint32_t)tid;
+        for (int r = 1; r < p.cluster; ++r) {
+          const uint32_t rb_addr = cluster_map(base, (uint32_t)r);
+          float v[M];
+#pragma unroll
+          for (int m = 0; m < M; ++m) v[m] = ld_cluster_f32(rb_addr + 4u * (uint32_t)(m * kRows));
+#pragma unroll
+          for (int m = 0; m < M; ++m) sum[m] += v[m];
+        }
+        if (n < p.N) {
+#pragma unroll
+          for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
+        }
+      }
+      cluster_sync_all();
+      break;  // a clustered CTA covers one row block
+    } else {
     if (seg_begin >= w0 && t_cur == T - 1) {
       if (n < p.N) {
 #pragma unroll
@@ -345,11 +397,27 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
         float sum[M];
 #pragma unroll
         for (int m = 0; m < M; ++m) sum[m] = 0.f;
-        for (int64_t i = i_first; i <= i_last; ++i) {
-          const int sl = (range_begin(i, p.W, p.G) / T == rb_cur) ? 0 : 1;
-          const float* src = p.ws + (i * 2 + sl) * (kRows * kMaxTokens);
+        // several contributors at a time: their loads are independent, the adds stay in
+        // CTA order
+        constexpr int kU = M <= 2 ? 8 : (M <= 8 ? 4 : 2);
+        for (int64_t i = i_first; i <= i_last; i += kU) {
+          float part[kU][M];
 #pragma unroll
-          for (int m = 0; m < M; ++m) sum[m] += __ldcg(src + m * kRows + tid);
+          for (int u = 0; u < kU; ++u) {
+            const int64_t ci = i + u;
+            if (ci <= i_last) {
+              const int sl = (range_begin(ci, p.W, p.G) / T == rb_cur) ? 0 : 1;
+              const float* src = p.ws + (ci * 2 + sl) * (kRows * kMaxTokens);
+#pragma unroll
+              for (int m = 0; m < M; ++m) part[u][m] = __ldcg(src + m * kRows + tid);
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < kU; ++u)
+            if (i + u <= i_last) {
+#pragma unroll
+              for (int m = 0; m < M; ++m) sum[m] += part[u][m];
+            }
         }
         if (n < p.N) {
 #pragma unroll
@@ -359,6 +427,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
       }
       named_bar_sync(1, kConsumerWarps * 32);
     }
+    }  // stream-K epilogue
 #pragma unroll
     for (int m = 0; m < M; ++m) acc[m] = 0.f;
   }
@@ -366,31 +435,43 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
 
 template <int M, int ES>
 sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem) {
-  auto kern = linear_cc_kernel<M, ES>;
-  static bool configured[kMaxDevices] = {};  // the smem opt-in is set once per device
+  auto kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
+  static bool configured[2][kMaxDevices] = {};  // kernel attributes, once per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
-  if (!configured[dev]) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess)
+  const int ci = p.cluster > 1 ? 1 : 0;
+  if (!configured[ci][dev]) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess ||
+        (ci && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
+      cudaGetLastError();
       return SP_ERR_CUDA;
-    configured[dev] = true;
+    }
+    configured[ci][dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)p.G);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int na = 1;
+  if (p.cluster > 1) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)p.cluster;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    na = 2;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = na;
   if (cudaLaunchKernelEx(&cfg, kern, p) != cudaSuccess) {
     cudaGetLastError();
     return SP_ERR_CUDA;
   }
-  return cudaGetLastError() == cudaSuccess ? SP_OK : SP_ERR_CUDA;
+  return SP_OK;
 }
 
 template <int ES>
@@ -416,6 +497,22 @@ sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem) {
   }
 }
 
+// Thread-block cluster split: each row block is split over S CTAs of one cluster
+// (S <= 16, S <= T, all CTAs within kCtasPerSm per SM), which replaces the global
+// split-K fix-up by a distributed-shared-memory reduction.  Taken when the clusters fill
+// at least 90% of the CTA slots, or when the matrix is small (few row blocks: there the
+// fixed latency of the global fix-up dominates); otherwise stream-K balances better.
+int cluster_cc(const sp_matrix* h) {
+  const int64_t cap = (int64_t)kCtasPerSm * h->num_sms;
+  const int64_t rb = std::max<int32_t>(h->RB, 1);
+  int64_t S = std::min<int64_t>(16, cap / rb);
+  S = std::min<int64_t>(S, h->T);
+  if (S < 2) return 1;
+  const bool fills = 10 * rb * S >= 9 * cap;
+  const bool small = 8 * rb <= cap;
+  return (fills || small) ? (int)S : 1;
+}
+
 int grid_cc(const sp_matrix* h) {
   const int64_t W = (int64_t)h->RB * h->T;
   static_assert(kCtasPerSm <= kMaxGridPerSm, "grid must fit the workspace counter region");
@@ -432,9 +529,10 @@ size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
 }
 
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool allow_cluster) {
+  const int S = allow_cluster ? cluster_cc(h) : 1;
   const size_t need = workspace_bytes_cc(h, M);
-  if (!ws || ws_bytes < need) return SP_ERR_WORKSPACE;
+  if (S == 1 && (!ws || ws_bytes < need)) return SP_ERR_WORKSPACE;
   LinearParams p{};
   p.buf = h->d_buf;
   p.off = h->d_off;
@@ -445,9 +543,10 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.T = h->T;
   p.RB = h->RB;
   p.W = (int64_t)h->RB * h->T;
-  p.G = grid_cc(h);
+  p.cluster = S;
+  p.G = S > 1 ? h->RB * S : grid_cc(h);
   p.cnt = reinterpret_cast<int*>(ws);
-  p.ws = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms));
+  p.ws = ws ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms)) : nullptr;
   p.timeout_ns = wait_timeout_ns();
   p.chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
   for (int64_t m0 = 0; m0 < M; m0 += kMaxTokens) {
@@ -456,11 +555,13 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.x = x + m0 * h->K;
     p.y = y + m0 * h->N;
     p.slot_bytes = p.chunk_region + (uint32_t)Mt * 128u;
-    // slots plus 2*slots mbarriers (<= 256 B) plus the flag must fit the budget
-    int slots = (int)std::min<size_t>(16, (kSmemBudget - 256 - 16) / p.slot_bytes);
+    // slots, 2*slots mbarriers (<= 256 B), the flag and (cluster mode) the FP32 partial
+    const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
+    int slots = (int)std::min<size_t>(16, (kSmemBudget - 256 - 16 - part_bytes) / p.slot_bytes);
     if (slots < 2) return SP_ERR_UNSUPPORTED;
     p.slots = slots;
-    const size_t smem = (size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16;
+    p.part_off = (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 15) / 16 * 16);
+    const size_t smem = p.part_off + part_bytes;
     const sp_status st = h->esize == 2 ? dispatch_m<2>(p, stream, smem) : dispatch_m<1>(p, stream, smem);
     if (st != SP_OK) return st;
   }

@@ -186,40 +186,50 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    if (lane == 0) {
-      const uint64_t pol = policy_evict_first();
-      const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
-      for (int64_t i = 0; i < n_pre; ++i) {  // weight bytes do not depend on the previous grid
-        const int64_t c = (w0 + i) % C;
-        const uint64_t o0 = p.off[c];
-        const uint32_t bytes = (uint32_t)(p.off[c + 1] - o0);
+    // The whole warp walks the items (it shares the offset window); lane 0 issues.
+    const uint64_t pol = policy_evict_first();
+    OffsetWindow ow;
+    ow.init(p.off, C + 1, w0 % C);
+    const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
+    for (int64_t i = 0; i < n_pre; ++i) {  // weight bytes do not depend on the previous grid
+      uint64_t o0, o1;
+      ow.at((w0 + i) % C, &o0, &o1);
+      if (lane == 0) {
+        const uint32_t bytes = (uint32_t)(o1 - o0);
         mbar_arrive_expect_tx(&full[i], bytes + tp.b_bytes);
         bulk_g2s_hint(smem + (size_t)i * p.slot_bytes + tp.chunk_off, p.buf + o0, bytes, &full[i], pol);
       }
-      pdl_wait();
-      pdl_launch_dependents();
-      int s = 0;
-      uint32_t ph = 0;
-      for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
-        const int64_t mtile = w / C;
-        const int64_t c = w % C;
-        const int t = (int)(c % T);
-        uint8_t* slot = smem + (size_t)s * p.slot_bytes;
-        if (n >= n_pre) {
+    }
+    pdl_wait();
+    pdl_launch_dependents();
+    int s = 0;
+    uint32_t ph = 0;
+    bool failed = false;
+    for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
+      const int64_t mtile = w / C;
+      const int64_t c = w % C;
+      const int t = (int)(c % T);
+      uint8_t* slot = smem + (size_t)s * p.slot_bytes;
+      if (n >= n_pre) {
+        uint64_t o0, o1;
+        ow.at(c, &o0, &o1);
+        if (lane == 0) {
           if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
             set_status(p.status, kStatusTimeout);
-            break;
+            failed = true;
+          } else {
+            const uint32_t bytes = (uint32_t)(o1 - o0);
+            mbar_arrive_expect_tx(&full[s], bytes + tp.b_bytes);
+            bulk_g2s_hint(slot + tp.chunk_off, p.buf + o0, bytes, &full[s], pol);
           }
-          const uint64_t o0 = p.off[c];
-          const uint32_t bytes = (uint32_t)(p.off[c + 1] - o0);
-          mbar_arrive_expect_tx(&full[s], bytes + tp.b_bytes);
-          bulk_g2s_hint(slot + tp.chunk_off, p.buf + o0, bytes, &full[s], pol);
         }
-        tma_load_2d(slot, &tmap_x, kTileK * t, (int)(mtile * tp.ntok), &full[s]);
-        if (++s == slots) {
-          s = 0;
-          ph ^= 1u;
-        }
+        failed = __shfl_sync(0xffffffffu, failed, 0);
+        if (failed) break;
+      }
+      if (lane == 0) tma_load_2d(slot, &tmap_x, kTileK * t, (int)(mtile * tp.ntok), &full[s]);
+      if (++s == slots) {
+        s = 0;
+        ph ^= 1u;
       }
     }
   } else if (warp == 1) {

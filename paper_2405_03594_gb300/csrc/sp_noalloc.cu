@@ -5,10 +5,10 @@
 // plugin or operator interface that owns every allocation) and are not allowed to
 // allocate device memory of their own; others run in latency-critical loops where a
 // cudaMalloc/cudaFree would synchronise the device.  They cannot provide the
-// workspace that sp_linear needs.  This entry point runs the same CUDA-core decode
-// kernel with the same launch configuration as sp_linear, but its scratch (the split-K
-// arrival counters and FP32 partials) lives in one fixed device array owned by the
-// library, so it never calls cudaMalloc, cudaFree or any allocating routine.
+// workspace that sp_linear needs.  This entry point runs the CUDA-core decode kernel in
+// its stream-K configuration, with its scratch (the split-K arrival counters and FP32
+// partials) in one fixed device array owned by the library, so it never calls
+// cudaMalloc, cudaFree or any allocating routine.
 //
 // The array is a file-scope __device__ variable: every GPU that loads libsp holds its
 // kNoAllocScratchBytes until the process exits.  In host code its name is only a
@@ -78,6 +78,7 @@ extern "C" sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, in
     cudaGetLastError();
     return SP_ERR_CUDA;
   }
+  // stream-K split-K with the partials and arrival counters in the static array
   return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), scratch,
-                          kNoAllocScratchBytes, (cudaStream_t)stream);
+                          kNoAllocScratchBytes, (cudaStream_t)stream, /*allow_cluster=*/false);
 }

@@ -25,8 +25,8 @@ D_MODEL = 4096
 D_FF = 11008
 # Initial weight scale of the stack: with N(0, 0.02^2) weights, 70% magnitude masks and
 # no normalisation, the gate*up product makes activations overflow within a few layers;
-# N(0, 0.004^2) keeps them O(10) through 32 layers.
-STACK_WEIGHT_STD = 0.004
+# N(0, 0.003^2) keeps them O(10) through 32 layers.
+STACK_WEIGHT_STD = 0.003
 
 
 def host_layer(pct: int, int8: bool, seed: int = 0, std: float = STACK_WEIGHT_STD):
