@@ -148,6 +148,15 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
 // A warp-wide window of 32 consecutive chunk offsets held one per lane, so that a
 // producer needs one coalesced global load per 31 chunks instead of a dependent L2
 // round trip per chunk.  Every lane of the warp must call at() with the same c.
+// Kept entries in chunk rows [0, 32q) -- the rows of the warps before warp quarter q of
+// a 128-row chunk: each lane sums its rows lane, lane + 32, ..., then one warp reduction
+// (a reduction per quarter would make the last warp of a chunk the slowest).
+__device__ __forceinline__ int kept_before_quarter(const uint64_t* masks, int q, int lane) {
+  int s = 0;
+  for (int k = 0; k < q; ++k) s += __popcll(masks[lane + 32 * k]);
+  return (int)__reduce_add_sync(0xffffffffu, (unsigned)s);
+}
+
 struct OffsetWindow {
   const uint64_t* off;
   int64_t n_off;  // entries in off[]

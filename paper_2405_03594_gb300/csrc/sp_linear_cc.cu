@@ -234,8 +234,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
         const int u = __shfl_up_sync(0xffffffffu, incl, d);
         if (lane >= d) incl += u;
       }
-      int base = 0;
-      for (int k = 0; k < warp; ++k) base += (int)__reduce_add_sync(0xffffffffu, __popcll(masks[lane + 32 * k]));
+      const int base = kept_before_quarter(masks, warp, lane);
       const int e0 = base + incl - pc;
 
       const uint16_t* xs = reinterpret_cast<const uint16_t*>(slot + p.chunk_region);
@@ -368,8 +367,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
           for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
         }
       }
-      cluster_sync_all();
-      break;  // a clustered CTA covers one row block
+      cluster_sync_all();  // a clustered CTA covers one row block: this was its last chunk
     } else {
     if (seg_begin >= w0 && t_cur == T - 1) {
       if (n < p.N) {

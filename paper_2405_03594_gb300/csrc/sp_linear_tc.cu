@@ -36,10 +36,10 @@ namespace {
 constexpr int kExpGroups = 2;         // expander warpgroups, taking alternate chunks
 constexpr int kThreads = (2 + 4 * kExpGroups) * 32;
 constexpr int kExpWarp0 = 2;          // first expander warp
-constexpr int kAStages = 4;           // A tiles in TMEM
+constexpr int kMaxAStages = 16;       // A tiles in TMEM (32 columns each), at most
+constexpr int kMaxDBufs = 2;          // D accumulators in TMEM (ntok columns each), at most
 constexpr int kMaxNtok = 256;         // tokens per tile (MMA N)
-constexpr uint32_t kTmemCols = 512;   // D (<= 256 columns) + kAStages x 32 columns
-constexpr uint32_t kACol0 = 256;
+constexpr uint32_t kTmemCols = 512;   // nD x D (ntok rounded to 32 columns) + nA x 32 A columns
 constexpr size_t kSmemLimit = 226 * 1024;
 constexpr int kMaxDevices = 64;
 constexpr int kMaxSlots = 16;
@@ -127,13 +127,92 @@ __device__ __forceinline__ uint16_t i8_to_bf16(uint32_t byte) {
   return (uint16_t)(__float_as_uint(f) >> 16);
 }
 
+// One output word (two adjacent columns) of a row's expansion, bf16 values: each kept
+// column takes the next value of the stream at shared address `pa` (which advances);
+// a dropped column gives +0.  Written in PTX so every column is one predicate-setting
+// AND, one predicated 16-bit shared load and one predicated pointer increment.
+template <uint32_t B0, uint32_t B1>
+__device__ __forceinline__ uint32_t expand_word_bf16(uint32_t m, uint32_t& pa) {
+  uint32_t o;
+  asm("{\n\t.reg .pred p0, p1;\n\t.reg .b32 t0, t1, lo, hi;\n\t"
+      "and.b32 t0, %2, %3;\n\t"
+      "setp.ne.b32 p0, t0, 0;\n\t"
+      "and.b32 t1, %2, %4;\n\t"
+      "setp.ne.b32 p1, t1, 0;\n\t"
+      "mov.b32 lo, 0;\n\t"
+      "mov.b32 hi, 0;\n\t"
+      "@p0 ld.shared.u16 lo, [%1];\n\t"
+      "@p0 add.u32 %1, %1, 2;\n\t"
+      "@p1 ld.shared.u16 hi, [%1];\n\t"
+      "@p1 add.u32 %1, %1, 2;\n\t"
+      "prmt.b32 %0, lo, hi, 0x5410;\n\t}"
+      : "=r"(o), "+r"(pa)
+      : "r"(m), "n"(B0), "n"(B1));
+  return o;
+}
+// The same for int8 values (one byte each), converted exactly to bf16.
+template <uint32_t B0, uint32_t B1>
+__device__ __forceinline__ uint32_t expand_word_i8(uint32_t m, uint32_t& pa) {
+  uint32_t lo = 0, hi = 0;
+  uint32_t b0, b1;
+  asm("{\n\t.reg .pred p0, p1;\n\t.reg .b32 t0, t1;\n\t"
+      "and.b32 t0, %3, %4;\n\t"
+      "setp.ne.b32 p0, t0, 0;\n\t"
+      "and.b32 t1, %3, %5;\n\t"
+      "setp.ne.b32 p1, t1, 0;\n\t"
+      "mov.b32 %0, 128;\n\t"
+      "mov.b32 %1, 128;\n\t"
+      "@p0 ld.shared.u8 %0, [%2];\n\t"
+      "@p0 add.u32 %2, %2, 1;\n\t"
+      "@p1 ld.shared.u8 %1, [%2];\n\t"
+      "@p1 add.u32 %2, %2, 1;\n\t}"
+      : "=r"(b0), "=r"(b1), "+r"(pa)
+      : "r"(m), "n"(B0), "n"(B1));
+  // a dropped column loads the byte 0x80 = -128 ... replaced below by +0
+  lo = (m & B0) ? i8_to_bf16(b0) : 0u;
+  hi = (m & B1) ? i8_to_bf16(b1) : 0u;
+  return lo | (hi << 16);
+}
+
+template <int ES, int I>
+__device__ __forceinline__ void expand_pair(uint32_t mlo, uint32_t mhi, uint32_t& pa, uint32_t& pb,
+                                            uint32_t (&o)[32]) {
+  constexpr uint32_t B0 = 1u << (2 * I), B1 = 1u << (2 * I + 1);
+  if constexpr (ES == 2) {
+    o[I] = expand_word_bf16<B0, B1>(mlo, pa);
+    o[16 + I] = expand_word_bf16<B0, B1>(mhi, pb);
+  } else {
+    o[I] = expand_word_i8<B0, B1>(mlo, pa);
+    o[16 + I] = expand_word_i8<B0, B1>(mhi, pb);
+  }
+  if constexpr (I + 1 < 16) expand_pair<ES, I + 1>(mlo, mhi, pa, pb, o);
+}
+
 struct TcParams {
   LinearParams p;     // shared fields (buf, off, scale, y, ws, cnt, status, N, K, T, RB, M, W, G, slots, ...)
   int32_t ntok;       // tokens per tile (MMA N), multiple of 16, <= 256
   int32_t mt;         // token tiles
   uint32_t b_bytes;   // bytes of one x tile in shared memory (ntok * 128)
   uint32_t chunk_off; // offset of the chunk region inside a slot
+  int32_t n_a;        // A stages in TMEM (2..kMaxAStages)
+  int32_t n_d;        // D buffers in TMEM (1..kMaxDBufs); segment k accumulates in buffer k % n_d
+  uint32_t d_cols;    // TMEM columns per D buffer (ntok rounded up to 32)
+  uint32_t a_col0;    // first TMEM column of the A stages (n_d * d_cols)
 };
+
+// TMEM split for a token tile of ntok columns: D buffers first, A stages after.  Small
+// tiles (decode) leave room for two D buffers and up to 14 A stages, so neither the
+// epilogue of one (row block, token tile) segment nor the tcgen05.commit round trip that
+// frees an A stage stalls the MMA issuer.
+__host__ __device__ inline void tmem_split(int ntok, int* n_a, int* n_d, uint32_t* d_cols) {
+  const uint32_t dc = ((uint32_t)ntok + 31u) / 32u * 32u;
+  const int nd = (2u * dc <= kTmemCols / 2) ? 2 : 1;
+  int na = (int)((kTmemCols - (uint32_t)nd * dc) / 32u);
+  if (na > kMaxAStages) na = kMaxAStages;
+  *n_a = na;
+  *n_d = nd;
+  *d_cols = dc;
+}
 
 template <int ES>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -145,12 +224,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)slots * p.slot_bytes);
   uint64_t* empty = full + slots;
   uint64_t* a_full = empty + slots;
-  uint64_t* a_empty = a_full + kAStages;
-  // D handshakes, one pair per expander warpgroup: a group's epilogues are sequential,
-  // so each group's parity waits never alias an older phase.
-  uint64_t* d_full = a_empty + kAStages;   // [kExpGroups]
-  uint64_t* d_empty = d_full + kExpGroups; // [kExpGroups]
-  uint32_t* tmem_base_slot = reinterpret_cast<uint32_t*>(d_empty + kExpGroups);
+  uint64_t* a_empty = a_full + kMaxAStages;
+  // D handshakes.  Segment k (the k-th (token tile, row block) this CTA touches)
+  // accumulates in buffer k % n_d, and its epilogue is run by the warpgroup that expanded
+  // its last K-tile.  d_full has one barrier per (buffer, warpgroup): a group waits on
+  // its own barriers one segment at a time, in order, so a parity wait can never match
+  // an older phase (a group may reach the end of a short segment before the MMA issuer
+  // has finished the previous segment on that buffer).  d_empty has one barrier per
+  // buffer: the MMA issuer starts segment k only after the epilogue of segment k - n_d
+  // has read that buffer, so those epilogues complete in order.
+  uint64_t* d_full = a_empty + kMaxAStages;               // [kMaxDBufs][kExpGroups]
+  uint64_t* d_empty = d_full + kMaxDBufs * kExpGroups;    // [kMaxDBufs]
+  uint32_t* tmem_base_slot = reinterpret_cast<uint32_t*>(d_empty + kMaxDBufs);
   volatile int* s_flag = reinterpret_cast<volatile int*>(tmem_base_slot + 1);  // one per warpgroup
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -164,14 +249,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 4 + 1);  // four expander warps + one MMA commit
     }
-    for (int a = 0; a < kAStages; ++a) {
+    for (int a = 0; a < kMaxAStages; ++a) {
       mbar_init(&a_full[a], 4);
       mbar_init(&a_empty[a], 1);
     }
-    for (int g = 0; g < kExpGroups; ++g) {
-      mbar_init(&d_full[g], 1);
-      mbar_init(&d_empty[g], 4);
-    }
+    for (int b = 0; b < kMaxDBufs * kExpGroups; ++b) mbar_init(&d_full[b], 1);
+    for (int b = 0; b < kMaxDBufs; ++b) mbar_init(&d_empty[b], 4);  // the epilogue warpgroup's four warps
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -189,11 +272,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The whole warp walks the items (it shares the offset window); lane 0 issues.
     const uint64_t pol = policy_evict_first();
     OffsetWindow ow;
-    ow.init(p.off, C + 1, w0 % C);
+    // item w = mtile * C + c, c = rb * T + t: walked with counters (no 64-bit division
+    // on the issuing thread's critical path)
+    int64_t c = w0 % C, mtile = w0 / C;
+    int t = (int)(c % T);
+    ow.init(p.off, C + 1, c);
     const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
-    for (int64_t i = 0; i < n_pre; ++i) {  // weight bytes do not depend on the previous grid
+    for (int64_t i = 0, ci = c; i < n_pre; ++i) {  // weight bytes do not depend on the previous grid
       uint64_t o0, o1;
-      ow.at((w0 + i) % C, &o0, &o1);
+      ow.at(ci, &o0, &o1);
+      if (++ci == C) ci = 0;
       if (lane == 0) {
         const uint32_t bytes = (uint32_t)(o1 - o0);
         mbar_arrive_expect_tx(&full[i], bytes + tp.b_bytes);
@@ -206,9 +294,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ph = 0;
     bool failed = false;
     for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
-      const int64_t mtile = w / C;
-      const int64_t c = w % C;
-      const int t = (int)(c % T);
       uint8_t* slot = smem + (size_t)s * p.slot_bytes;
       if (n >= n_pre) {
         uint64_t o0, o1;
@@ -231,6 +316,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         s = 0;
         ph ^= 1u;
       }
+      if (++t == T) t = 0;
+      if (++c == C) {
+        c = 0;
+        ++mtile;
+      }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -238,21 +328,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       pdl_wait();
       pdl_launch_dependents();
       const uint32_t idesc = idesc_bf16(tp.ntok);
+      const int n_a = tp.n_a, n_d = tp.n_d;
       int s = 0, as = 0;
       uint32_t ph = 0, aph = 0;
-      uint32_t dph[kExpGroups] = {};
-      int prev_group = -1;  // warpgroup that ran the previous segment's epilogue
+      int k = -1;  // local segment number
+      int db = 0;  // D buffer of segment k
+      uint32_t d_taddr = tmem;
       bool dead = false;
-      for (int64_t w = w0, n = 0; w < w1; ++w, ++n) {
-        const bool seg_first = (w == w0) || (w % T == 0);
-        const bool seg_last = (w + 1 == w1) || ((w + 1) % T == 0);
-        if (!dead && seg_first && prev_group >= 0) {
-          // D is reused: wait until that epilogue has read the previous segment
-          if (!mbar_wait(&d_empty[prev_group], dph[prev_group], p.timeout_ns)) {
-            dead = true;
-            set_status(p.status, kStatusTimeout);
+      int t = (int)(w0 % T);  // K-tile of item w
+      for (int64_t w = w0; w < w1; ++w) {
+        const bool seg_first = (w == w0) || t == 0;
+        const bool seg_last = (w + 1 == w1) || t == T - 1;
+        if (++t == T) t = 0;
+        if (seg_first) {
+          ++k;
+          db = k % n_d;
+          d_taddr = tmem + (uint32_t)db * tp.d_cols;
+          // D buffer reuse: wait for the (k / n_d - 1)-th completion of d_empty[db], the
+          // epilogue of segment k - n_d
+          if (!dead && k >= n_d) {
+            if (!mbar_wait(&d_empty[db], (uint32_t)((k / n_d - 1) & 1), p.timeout_ns)) {
+              dead = true;
+              set_status(p.status, kStatusTimeout);
+            }
           }
-          dph[prev_group] ^= 1u;
         }
         if (!dead && !mbar_wait(&full[s], ph, p.timeout_ns)) {
           dead = true;
@@ -265,22 +364,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!dead) {
           tc_fence_after();
           const uint32_t b_saddr = smem_u32(smem + (size_t)s * p.slot_bytes);
-          const uint32_t a_taddr = tmem + kACol0 + (uint32_t)as * 32u;
+          const uint32_t a_taddr = tmem + tp.a_col0 + (uint32_t)as * 32u;
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {
             const uint64_t bdesc = smem_desc_sw128(b_saddr + (uint32_t)kk * 32u);
-            mma_ts(tmem, a_taddr + (uint32_t)kk * 8u, bdesc, idesc, (seg_first && kk == 0) ? 0u : 1u);
+            mma_ts(d_taddr, a_taddr + (uint32_t)kk * 8u, bdesc, idesc, (seg_first && kk == 0) ? 0u : 1u);
           }
           mma_commit(&empty[s]);
           mma_commit(&a_empty[as]);
-          if (seg_last) mma_commit(&d_full[n % kExpGroups]);
+          if (seg_last) mma_commit(&d_full[db * kExpGroups + (int)((w - w0) % kExpGroups)]);
         }
-        if (seg_last) prev_group = (int)(n % kExpGroups);
         if (++s == slots) {
           s = 0;
           ph ^= 1u;
         }
-        if (++as == kAStages) {
+        if (++as == n_a) {
           as = 0;
           aph ^= 1u;
         }
@@ -296,16 +394,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const int tid128 = (warp - kExpWarp0 - 4 * grp) * 32 + lane;
     bool dead = false;
-    uint32_t dph = 0;  // phase of this group's own D handshake
+    const int n_a = tp.n_a;
     const int64_t sg_first = w0 / T;
+    // ring positions of item n = grp, grp + kExpGroups, ... (slots, n_a >= kExpGroups)
+    int s = grp, as = grp;
+    uint32_t ph = 0, aph = 0;
+    int t = (int)((w0 + grp) % T);  // K-tile of item w
+    uint32_t dph_bits = 0;          // phase parity of this group's d_full barrier, per buffer
     for (int64_t w = w0 + grp, n = grp; w < w1; w += kExpGroups, n += kExpGroups) {
-      const int s = (int)(n % slots);
-      const uint32_t ph = (uint32_t)((n / slots) & 1);
-      const int as = (int)(n % kAStages);
-      const uint32_t aph = (uint32_t)((n / kAStages) & 1);
+      const bool seg_last = (w + 1 == w1) || t == T - 1;
+      for (t += kExpGroups; t >= T;) t -= T;
       if (!dead) {
         bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
-        if (ok && n >= kAStages) ok = __all_sync(0xffffffffu, mbar_wait(&a_empty[as], aph ^ 1u, p.timeout_ns));
+        if (ok && n >= n_a) ok = __all_sync(0xffffffffu, mbar_wait(&a_empty[as], aph ^ 1u, p.timeout_ns));
         if (!ok) {
           dead = true;
           set_status(p.status, kStatusTimeout);
@@ -325,8 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int u = __shfl_up_sync(0xffffffffu, incl, d);
           if (lane >= d) incl += u;
         }
-        int base = 0;
-        for (int k = 0; k < q; ++k) base += (int)__reduce_add_sync(0xffffffffu, __popcll(masks[lane + 32 * k]));
+        const int base = kept_before_quarter(masks, q, lane);
         const int e0 = base + incl - pc;
         // Static walk over the 64 columns: a kept column takes the next value of its
         // half's stream.  Columns 0-31 and 32-63 read two independent streams (the
@@ -334,34 +434,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         // parallelism; each step is one predicate-setting AND, a predicated load and a
         // predicated pointer increment.
         uint32_t o[32];
-        if (ES == 2) {
-          const uint16_t* va = reinterpret_cast<const uint16_t*>(chunk + kMaskBytes) + e0;
-          const uint16_t* vb = va + plo;
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            uint32_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;
-            if (mlo & (1u << (2 * i))) a0 = *va++;
-            if (mhi & (1u << (2 * i))) b0 = *vb++;
-            if (mlo & (1u << (2 * i + 1))) a1 = *va++;
-            if (mhi & (1u << (2 * i + 1))) b1 = *vb++;
-            o[i] = __byte_perm(a0, a1, 0x5410);
-            o[16 + i] = __byte_perm(b0, b1, 0x5410);
-          }
-        } else {
-          const uint8_t* va = chunk + kMaskBytes + e0;
-          const uint8_t* vb = va + plo;
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            uint32_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;
-            if (mlo & (1u << (2 * i))) a0 = i8_to_bf16(*va++);
-            if (mhi & (1u << (2 * i))) b0 = i8_to_bf16(*vb++);
-            if (mlo & (1u << (2 * i + 1))) a1 = i8_to_bf16(*va++);
-            if (mhi & (1u << (2 * i + 1))) b1 = i8_to_bf16(*vb++);
-            o[i] = __byte_perm(a0, a1, 0x5410);
-            o[16 + i] = __byte_perm(b0, b1, 0x5410);
-          }
-        }
-        tmem_store32(tmem + lane_base + kACol0 + (uint32_t)as * 32u, o);
+        const uint32_t vbase = smem_u32(chunk + kMaskBytes);
+        uint32_t pa = vbase + (uint32_t)(e0 * ES);   // stream of columns 0-31
+        uint32_t pb = pa + (uint32_t)(plo * ES);     // stream of columns 32-63
+        expand_pair<ES, 0>(mlo, mhi, pa, pb, o);
+        tmem_store32(tmem + lane_base + tp.a_col0 + (uint32_t)as * 32u, o);
         tmem_store_wait();
       }
       tc_fence_before();
@@ -370,10 +447,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(&a_full[as]);
         mbar_arrive(&empty[s]);
       }
+      if ((s += kExpGroups) >= slots) {
+        s -= slots;
+        ph ^= 1u;
+      }
+      if ((as += kExpGroups) >= n_a) {
+        as -= n_a;
+        aph ^= 1u;
+      }
 
       // ---------------------------------------------------------- segment end: epilogue
       // Taken by the warpgroup that expanded the segment's last K-tile.
-      const bool seg_last = (w + 1 == w1) || ((w + 1) % T == 0);
       if (!seg_last) continue;
       const int64_t sg = w / T;  // segment = (token tile, row block)
       const int64_t seg_begin = sg * T;
@@ -381,14 +465,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t rb = sg % p.RB;
       const int64_t nrow = rb * kRows + r;
       const float sc = (ES == 1 && nrow < p.N) ? p.scale[nrow] : 1.f;
+      const int kseg = (int)(sg - sg_first);  // local segment number
+      const int db = kseg % tp.n_d;
+      const uint32_t dph = (dph_bits >> db) & 1u;
+      dph_bits ^= 1u << db;
+      const uint32_t d_taddr = tmem + (uint32_t)db * tp.d_cols;
       if (!dead) {
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&d_full[grp], dph, p.timeout_ns));
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&d_full[db * kExpGroups + grp], dph, p.timeout_ns));
         if (!ok) {
           dead = true;
           set_status(p.status, kStatusTimeout);
         }
       }
-      dph ^= 1u;
       tc_fence_after();
       // this CTA ran the whole segment: its first and its last K-tile
       const bool complete = seg_begin >= w0 && (w + 1) % T == 0;
@@ -398,7 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c0 = 0; c0 < tp.ntok; c0 += 32) {
         uint32_t v[32];
         if (!dead) {
-          tmem_load32(tmem + lane_base + (uint32_t)c0, v);
+          tmem_load32(d_taddr + lane_base + (uint32_t)c0, v);
           tmem_load_wait();
         }
 #pragma unroll
@@ -415,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&d_empty[grp]);
+      if (lane == 0) mbar_arrive(&d_empty[db]);
       if (!complete) {
         const int bar = 1 + grp;
         __threadfence();
@@ -560,12 +648,15 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.cnt = reinterpret_cast<int*>(ws);
   p.ws = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms));
   p.timeout_ns = wait_timeout_ns();
+  tmem_split(tp.ntok, &tp.n_a, &tp.n_d, &tp.d_cols);
+  tp.a_col0 = (uint32_t)tp.n_d * tp.d_cols;
   tp.b_bytes = (uint32_t)tp.ntok * 128u;
   tp.chunk_off = (tp.b_bytes + 1023u) / 1024u * 1024u;
   p.chunk_region = (uint32_t)((h->max_chunk + 1023) / 1024 * 1024);
   p.slot_bytes = tp.chunk_off + p.chunk_region;
   // base alignment + barriers (2 per slot, 2 per A stage, 2 for D), TMEM address, flag
-  const size_t tail = 1024 + 8 * (2 * kMaxSlots + 2 * kAStages + 2 * kExpGroups) + 4 + 4 * kExpGroups + 16;
+  const size_t tail =
+      1024 + 8 * (2 * kMaxSlots + 2 * kMaxAStages + kMaxDBufs * (kExpGroups + 1)) + 4 + 4 * kExpGroups + 16;
   const int slots = (int)std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes);
   if (slots < 2) return SP_ERR_UNSUPPORTED;
   p.slots = slots;

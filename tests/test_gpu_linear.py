@@ -209,6 +209,18 @@ def test_config_sweep_nonuniform_sampled(sp, oracle, name, pct):
     sp.check()
 
 
+@pytest.mark.parametrize("N,K", [(4096, 64), (2000, 128), (1500, 200), (700, 1024)])
+@pytest.mark.parametrize("M", [17, 100, 256, 300])
+def test_tensor_core_short_segments(sp, oracle, N, K, M):
+    """Tensor-core path with few K-tiles per row block (T = 1 .. 16): every CTA's range
+    covers many short (token tile, row block) segments, so an expander warpgroup can
+    finish a segment before the MMA issuer has finished the previous one on the same
+    accumulator; wide token tiles (up to 256 tokens) and a ragged last token tile."""
+    vals, s, mask, x = _case(N, K, M, 70, seed=N + K + M)
+    _, y = _run(sp, vals, s, mask, x, "tensor_core")
+    gu.assert_close(gu.bf16_from_dev(y), _ref(oracle, vals, s, mask, x), f"{N}x{K} M={M}")
+
+
 def test_shared_workspace_across_grids(sp, oracle):
     """Matrices whose launches use different grid sizes share one workspace, interleaved:
     the split-K counters must never be overlaid by another call's partials."""
