@@ -67,6 +67,7 @@ struct LinearParams {
   int32_t cluster;      // CUDA-core kernel: > 1 = split each row block over this many CTAs of
                         // one thread-block cluster; <= 1 = stream-K over the workspace
   uint32_t part_off;    // cluster mode: shared-memory offset of the CTA's FP32 partial
+  uint32_t comb_off;    // warp-per-chunk kernel: shared-memory offset of the warps' partials
 };
 
 // Workspace layout, fixed per device so that calls with different grids can share it:

@@ -99,6 +99,293 @@ struct Stream16 {
   }
 };
 
+// CTA's work items [w0, w1): a contiguous run of chunks (stream-K), or -- in cluster
+// mode -- K-tiles [r*T/S, (r+1)*T/S) of the row block of its cluster (r = its rank).
+__device__ __forceinline__ void cta_range(const LinearParams& p, bool clustered, int64_t* w0, int64_t* w1,
+                                          uint32_t* crank) {
+  if (clustered) {
+    const int64_t seg = blockIdx.x / p.cluster;
+    *crank = cluster_rank();
+    *w0 = seg * p.T + (int64_t)*crank * p.T / p.cluster;
+    *w1 = seg * p.T + (int64_t)(*crank + 1) * p.T / p.cluster;
+  } else {
+    *crank = 0;
+    *w0 = range_begin(blockIdx.x, p.W, p.G);
+    *w1 = range_begin(blockIdx.x + 1, p.W, p.G);
+  }
+}
+
+// Producer warp: one cp.async.bulk per chunk (evict-first L2 hint) plus one copy of
+// x[m, 64t : 64t+64) per batch row into ring slot n % slots, in item order.  The whole
+// warp walks the chunk list (it shares the offset window); lane 0 issues.  Weight bytes
+// do not depend on the previous kernel in the stream: the first ring fill is issued
+// before griddepcontrol.wait; every x copy comes after it.
+template <int M>
+__device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, uint64_t* full, uint64_t* empty,
+                                        int64_t w0, int64_t w1, int lane) {
+  const int T = p.T;
+  const int slots = p.slots;
+  const uint64_t pol = policy_evict_first();
+  OffsetWindow ow;
+  ow.init(p.off, p.W + 1, w0);
+  const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
+  {
+    int t = (int)(w0 % T);
+    for (int64_t i = 0; i < n_pre; ++i) {
+      uint64_t o0, o1;
+      ow.at(w0 + i, &o0, &o1);
+      if (lane == 0) {
+        const uint32_t bytes = (uint32_t)(o1 - o0);
+        const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
+        mbar_arrive_expect_tx(&full[i], bytes + (uint32_t)M * (uint32_t)valid * 2u);
+        bulk_g2s_hint(smem + (size_t)i * p.slot_bytes, p.buf + o0, bytes, &full[i], pol);
+      }
+      if (++t == T) t = 0;
+    }
+  }
+  pdl_wait();
+  pdl_launch_dependents();
+  int s = 0;
+  uint32_t ph = 0;
+  int t = (int)(w0 % T);
+  int64_t n_issued = 0;
+  bool failed = false;
+  for (int64_t w = w0; w < w1 && !failed; ++w, ++n_issued) {
+    const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
+    const uint32_t xb = (uint32_t)valid * 2u;
+    uint8_t* slot = smem + (size_t)s * p.slot_bytes;
+    if (n_issued >= n_pre) {
+      uint64_t o0, o1;
+      ow.at(w, &o0, &o1);
+      if (lane == 0) {
+        if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+          set_status(p.status, kStatusTimeout);
+          failed = true;
+        } else {
+          const uint32_t bytes = (uint32_t)(o1 - o0);
+          mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
+          bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
+        }
+      }
+      failed = __shfl_sync(0xffffffffu, failed, 0);
+      if (failed) break;
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int m = 0; m < M; ++m)
+        bulk_g2s(slot + p.chunk_region + m * 128, p.x + (int64_t)m * p.K + (int64_t)kTileK * t, xb, &full[s]);
+    }
+    if (++t == T) t = 0;
+    if (++s == slots) {
+      s = 0;
+      ph ^= 1u;
+    }
+  }
+}
+
+// x of one chunk's K-tile as shuffle sources: lane j holds x[m, 64t+j] (XL) and
+// x[m, 64t+32+j] (XH), two batch rows per register.
+template <int M>
+__device__ __forceinline__ void load_x(const uint8_t* slot, uint32_t chunk_region, int lane,
+                                       uint32_t (&XL)[(M + 1) / 2], uint32_t (&XH)[(M + 1) / 2]) {
+  const uint16_t* xs = reinterpret_cast<const uint16_t*>(slot + chunk_region);
+#pragma unroll
+  for (int q = 0; q < (M + 1) / 2; ++q) {
+    const uint32_t a0 = xs[(2 * q) * 64 + lane], b0 = xs[(2 * q) * 64 + 32 + lane];
+    const uint32_t a1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + lane] : 0u;
+    const uint32_t b1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + 32 + lane] : 0u;
+    XL[q] = a0 | (a1 << 16);
+    XH[q] = b0 | (b1 << 16);
+  }
+}
+
+// acc[m] += sum over the kept columns j of one chunk row of value(j) * x[m, 64t+j].
+// The row's 64-bit mask (lo, hi) splits into two 32-column halves walked as two
+// independent chains, each from its highest set bit down (bfind), consuming that
+// half's values from the top; the x operand comes by shuffle from lane j % 32.  `e0`
+// is the index of the row's first value in the chunk's packed values; plo / pc are the
+// kept counts of the low half / the row.  Every lane of the warp calls this together.
+template <int M, int ES>
+__device__ __forceinline__ void row_dot(uint32_t lo, uint32_t hi, int plo, int pc, int e0, const uint8_t* vals,
+                                        const uint32_t (&XL)[(M + 1) / 2], const uint32_t (&XH)[(M + 1) / 2],
+                                        float (&acc)[M]) {
+  constexpr int MP = (M + 1) / 2;
+  const int top_lo = e0 + plo - 1;  // highest-column value of the low half
+  const int top_hi = e0 + pc - 1;   // ... of the high half
+  const int iters = (int)__reduce_max_sync(0xffffffffu, (unsigned)max(plo, pc - plo));
+  if constexpr (ES == 2 && M <= 4) {
+    // bf16, small batch: two chain steps per loop trip share one word load per chain,
+    // and each chain keeps its own accumulators
+    float accl[M], acch[M];
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      accl[m] = 0.f;
+      acch[m] = 0.f;
+    }
+    Stream16 sl, sh;
+    const uint32_t vbase = smem_u32(vals);
+    sl.init(vbase + 2u * (uint32_t)top_lo);
+    sh.init(vbase + 2u * (uint32_t)top_hi);
+    for (int q = 0; q < iters; q += 2) {
+      const uint32_t wl = sl.next_pair(), wh = sh.next_pair();
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int jl = msb32(lo), jh = msb32(hi);
+        lo = clear_bit(lo, jl);
+        hi = clear_bit(hi, jh);
+        const uint16_t vl = h == 0 ? hi16(wl) : lo16(wl);
+        const uint16_t vh = h == 0 ? hi16(wh) : lo16(wh);
+#pragma unroll
+        for (int r = 0; r < MP; ++r) {
+          const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+          const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+          if (jl >= 0) {
+            accl[2 * r] = fma_bf16(vl, lo16(xl), accl[2 * r]);
+            if (2 * r + 1 < M) accl[2 * r + 1] = fma_bf16(vl, hi16(xl), accl[2 * r + 1]);
+          }
+          if (jh >= 0) {
+            acch[2 * r] = fma_bf16(vh, lo16(xh), acch[2 * r]);
+            if (2 * r + 1 < M) acch[2 * r + 1] = fma_bf16(vh, hi16(xh), acch[2 * r + 1]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < M; ++m) acc[m] += accl[m] + acch[m];
+  } else {
+    // larger batches (or int8 values): one value per chain step, one accumulator set
+#pragma unroll 2
+    for (int q = 0; q < iters; ++q) {
+      const int jl = msb32(lo), jh = msb32(hi);
+      lo = clear_bit(lo, jl);
+      hi = clear_bit(hi, jh);
+      uint16_t wl = 0, wh = 0;
+      if (ES == 2) {
+        if (jl >= 0) wl = reinterpret_cast<const uint16_t*>(vals)[top_lo - q];
+        if (jh >= 0) wh = reinterpret_cast<const uint16_t*>(vals)[top_hi - q];
+      } else {
+        if (jl >= 0) wl = i8_to_bf16(vals[top_lo - q]);
+        if (jh >= 0) wh = i8_to_bf16(vals[top_hi - q]);
+      }
+#pragma unroll
+      for (int r = 0; r < MP; ++r) {
+        const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+        const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+        if (jl >= 0) {
+          acc[2 * r] = fma_bf16(wl, lo16(xl), acc[2 * r]);
+          if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wl, hi16(xl), acc[2 * r + 1]);
+        }
+        if (jh >= 0) {
+          acc[2 * r] = fma_bf16(wh, lo16(xh), acc[2 * r]);
+          if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wh, hi16(xh), acc[2 * r + 1]);
+        }
+      }
+    }
+  }
+}
+
+// End of row block rb for consumer thread tid <-> output row rb*128 + tid, holding this
+// CTA's FP32 sums `acc` over the row block's K-tiles it covered.
+//  cluster mode: each CTA leaves its partial in its own shared memory; after a cluster
+//    barrier rank 0 adds the other ranks' partials in rank order (distributed shared
+//    memory) and writes y; a second barrier keeps every partial alive until then.
+//  stream-K: a CTA that covered the whole row block (`complete`) writes y; otherwise it
+//    stores its partial in workspace slot `my_slot` (0 = its first row block, 1 = its
+//    last), and the last of the row block's CTAs to arrive sums the partials in CTA
+//    order (deterministic) and writes y.
+// All consumer threads (kConsumerWarps warps) call this together.
+template <int M, int ES, bool CL>
+__device__ __forceinline__ void row_block_end(const LinearParams& p, uint8_t* smem, volatile int* s_flag,
+                                              const float (&acc)[M], int64_t rb, bool complete, int my_slot,
+                                              uint32_t crank, int tid) {
+  const int T = p.T;
+  const int64_t seg_begin = rb * T;
+  const int64_t n = rb * kRows + tid;
+  const float sc = (ES == 1 && n < p.N) ? p.scale[n] : 1.f;
+  if constexpr (CL) {
+    float* part = reinterpret_cast<float*>(smem + p.part_off);
+#pragma unroll
+    for (int m = 0; m < M; ++m) part[m * kRows + tid] = acc[m];
+    cluster_sync_all();
+    if (crank == 0) {
+      float sum[M];
+#pragma unroll
+      for (int m = 0; m < M; ++m) sum[m] = acc[m];
+      const uint32_t base = smem_u32(part) + 4u * (uint32_t)tid;
+      for (int r = 1; r < p.cluster; ++r) {
+        const uint32_t rb_addr = cluster_map(base, (uint32_t)r);
+        float v[M];
+#pragma unroll
+        for (int m = 0; m < M; ++m) v[m] = ld_cluster_f32(rb_addr + 4u * (uint32_t)(m * kRows));
+#pragma unroll
+        for (int m = 0; m < M; ++m) sum[m] += v[m];
+      }
+      if (n < p.N) {
+#pragma unroll
+        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
+      }
+    }
+    cluster_sync_all();
+  } else if (complete) {
+    if (n < p.N) {
+#pragma unroll
+      for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(acc[m] * sc);
+    }
+  } else {
+    float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * (kRows * kMaxTokens);
+#pragma unroll
+    for (int m = 0; m < M; ++m) __stcg(wsp + m * kRows + tid, acc[m]);
+    __threadfence();
+    named_bar_sync(1, kConsumerWarps * 32);
+    const int64_t i_first = owner_of(seg_begin, p.W, p.G);
+    const int64_t i_last = owner_of(seg_begin + T - 1, p.W, p.G);
+    const int sf = (range_begin(i_first, p.W, p.G) / T == rb) ? 0 : 1;
+    int* ctr = p.cnt + i_first * 2 + sf;
+    if (tid == 0) {
+      const int old = atomicAdd(ctr, 1);
+      *s_flag = (old == (int)(i_last - i_first)) ? 1 : 0;
+    }
+    named_bar_sync(1, kConsumerWarps * 32);
+    if (*s_flag) {
+      __threadfence();
+      float sum[M];
+#pragma unroll
+      for (int m = 0; m < M; ++m) sum[m] = 0.f;
+      // several contributors at a time: their loads are independent, the adds stay in
+      // CTA order
+      constexpr int kU = M <= 2 ? 8 : (M <= 8 ? 4 : 2);
+      for (int64_t i = i_first; i <= i_last; i += kU) {
+        float part[kU][M];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int64_t ci = i + u;
+          if (ci <= i_last) {
+            const int sl = (range_begin(ci, p.W, p.G) / T == rb) ? 0 : 1;
+            const float* src = p.ws + (ci * 2 + sl) * (kRows * kMaxTokens);
+#pragma unroll
+            for (int m = 0; m < M; ++m) part[u][m] = __ldcg(src + m * kRows + tid);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u)
+          if (i + u <= i_last) {
+#pragma unroll
+            for (int m = 0; m < M; ++m) sum[m] += part[u][m];
+          }
+      }
+      if (n < p.N) {
+#pragma unroll
+        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
+      }
+      if (tid == 0) atomicExch(ctr, 0);
+    }
+    named_bar_sync(1, kConsumerWarps * 32);
+  }
+}
+
+// Thread-per-row kernel (any M <= kMaxTokens): the four consumer warps share each chunk,
+// thread r owning row r; its first value is found by a popc prefix sum over the chunk's
+// masks (warp scan plus the other warps' kept counts).
 template <int M, int ES, bool CL>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -108,19 +395,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
   const int T = p.T;
   const int slots = p.slots;
-  constexpr bool clustered = CL;  // split-K over a thread-block cluster (else stream-K)
   int64_t w0, w1;
-  uint32_t crank = 0;
-  if (clustered) {
-    // cluster c owns row block c; its CTA of rank r takes K-tiles [r*T/S, (r+1)*T/S)
-    const int64_t seg = blockIdx.x / p.cluster;
-    crank = cluster_rank();
-    w0 = seg * T + (int64_t)crank * T / p.cluster;
-    w1 = seg * T + (int64_t)(crank + 1) * T / p.cluster;
-  } else {
-    w0 = range_begin(blockIdx.x, p.W, p.G);
-    w1 = range_begin(blockIdx.x + 1, p.W, p.G);
-  }
+  uint32_t crank;
+  cta_range(p, CL, &w0, &w1, &crank);
 
   if (tid == 0) {
     for (int s = 0; s < slots; ++s) {
@@ -132,78 +409,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    // ------------------------------------------------------------ producer
-    // The whole warp walks the chunk list (it shares the offset window); lane 0 issues.
-    // Weight bytes do not depend on the previous kernel in the stream: the first ring
-    // fill is issued before griddepcontrol.wait; every x copy comes after it.
-    const uint64_t pol = policy_evict_first();
-    OffsetWindow ow;
-    ow.init(p.off, p.W + 1, w0);
-    const int64_t n_pre = imin64((int64_t)slots, w1 - w0);
-    {
-      int t = (int)(w0 % T);
-      for (int64_t i = 0; i < n_pre; ++i) {
-        uint64_t o0, o1;
-        ow.at(w0 + i, &o0, &o1);
-        if (lane == 0) {
-          const uint32_t bytes = (uint32_t)(o1 - o0);
-          const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
-          mbar_arrive_expect_tx(&full[i], bytes + (uint32_t)M * (uint32_t)valid * 2u);
-          bulk_g2s_hint(smem + (size_t)i * p.slot_bytes, p.buf + o0, bytes, &full[i], pol);
-        }
-        if (++t == T) t = 0;
-      }
-    }
-    pdl_wait();
-    pdl_launch_dependents();
-    int s = 0;
-    uint32_t ph = 0;
-    int t = (int)(w0 % T);
-    int64_t n_issued = 0;
-    bool failed = false;
-    for (int64_t w = w0; w < w1 && !failed; ++w, ++n_issued) {
-      const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
-      const uint32_t xb = (uint32_t)valid * 2u;
-      uint8_t* slot = smem + (size_t)s * p.slot_bytes;
-      if (n_issued >= n_pre) {
-        uint64_t o0, o1;
-        ow.at(w, &o0, &o1);
-        if (lane == 0) {
-          if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
-            set_status(p.status, kStatusTimeout);
-            failed = true;
-          } else {
-            const uint32_t bytes = (uint32_t)(o1 - o0);
-            mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
-            bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
-          }
-        }
-        failed = __shfl_sync(0xffffffffu, failed, 0);
-        if (failed) break;
-      }
-      if (lane == 0) {
-#pragma unroll
-        for (int m = 0; m < M; ++m)
-          bulk_g2s(slot + p.chunk_region + m * 128, p.x + (int64_t)m * p.K + (int64_t)kTileK * t, xb, &full[s]);
-      }
-      if (++t == T) t = 0;
-      if (++s == slots) {
-        s = 0;
-        ph ^= 1u;
-      }
-    }
+    produce<M>(p, smem, full, empty, w0, w1, lane);
     return;
   }
 
   // -------------------------------------------------------------- consumers
   pdl_wait();  // y, the workspace and x belong to the stream order
   pdl_launch_dependents();
-  // Thread r owns row r of every chunk.  Its 64-bit mask splits into two 32-column
-  // halves walked as two independent chains, each from its highest set bit down
-  // (bfind), consuming that half's values from the top.  Lane j holds x[m, 64t+j]
-  // (low half) and x[m, 64t+32+j] (high half), two batch rows per register, and the
-  // other lanes fetch them by shuffle.
-  constexpr int MP = (M + 1) / 2;
   float acc[M];
 #pragma unroll
   for (int m = 0; m < M; ++m) acc[m] = 0.f;
@@ -226,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
       const uint8_t* slot = smem + (size_t)s * p.slot_bytes;
       const uint64_t* masks = reinterpret_cast<const uint64_t*>(slot);
       const uint64_t mk = masks[tid];
-      uint32_t lo = (uint32_t)mk, hi = (uint32_t)(mk >> 32);
+      const uint32_t lo = (uint32_t)mk, hi = (uint32_t)(mk >> 32);
       const int plo = __popc(lo), pc = plo + __popc(hi);
       int incl = pc;
 #pragma unroll
@@ -235,93 +447,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
         if (lane >= d) incl += u;
       }
       const int base = kept_before_quarter(masks, warp, lane);
-      const int e0 = base + incl - pc;
-
-      const uint16_t* xs = reinterpret_cast<const uint16_t*>(slot + p.chunk_region);
-      uint32_t XL[MP], XH[MP];
-#pragma unroll
-      for (int q = 0; q < MP; ++q) {
-        const uint32_t a0 = xs[(2 * q) * 64 + lane], b0 = xs[(2 * q) * 64 + 32 + lane];
-        const uint32_t a1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + lane] : 0u;
-        const uint32_t b1 = (2 * q + 1 < M) ? xs[(2 * q + 1) * 64 + 32 + lane] : 0u;
-        XL[q] = a0 | (a1 << 16);
-        XH[q] = b0 | (b1 << 16);
-      }
-      const uint8_t* vals = slot + kMaskBytes;
-      const int top_lo = e0 + plo - 1;  // highest-column value of the low half
-      const int top_hi = e0 + pc - 1;   // ... of the high half
-      const int iters = (int)__reduce_max_sync(0xffffffffu, (unsigned)max(plo, pc - plo));
-      float accl[M <= 4 ? M : 1], acch[M <= 4 ? M : 1];
-#pragma unroll
-      for (int m = 0; m < (M <= 4 ? M : 1); ++m) {
-        accl[m] = 0.f;
-        acch[m] = 0.f;
-      }
-      if (ES == 2 && M <= 4) {
-        // bf16, small batch: two chain steps per loop trip share one word load per chain,
-        // and each chain keeps its own accumulators
-        Stream16 sl, sh;
-        const uint32_t vbase = smem_u32(vals);
-        sl.init(vbase + 2u * (uint32_t)top_lo);
-        sh.init(vbase + 2u * (uint32_t)top_hi);
-        for (int q = 0; q < iters; q += 2) {
-          const uint32_t wl = sl.next_pair(), wh = sh.next_pair();
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int jl = msb32(lo), jh = msb32(hi);
-            lo = clear_bit(lo, jl);
-            hi = clear_bit(hi, jh);
-            const uint16_t vl = h == 0 ? hi16(wl) : lo16(wl);
-            const uint16_t vh = h == 0 ? hi16(wh) : lo16(wh);
-#pragma unroll
-            for (int r = 0; r < MP; ++r) {
-              const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
-              const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
-              if (jl >= 0) {
-                accl[2 * r] = fma_bf16(vl, lo16(xl), accl[2 * r]);
-                if (2 * r + 1 < M) accl[2 * r + 1] = fma_bf16(vl, hi16(xl), accl[2 * r + 1]);
-              }
-              if (jh >= 0) {
-                acch[2 * r] = fma_bf16(vh, lo16(xh), acch[2 * r]);
-                if (2 * r + 1 < M) acch[2 * r + 1] = fma_bf16(vh, hi16(xh), acch[2 * r + 1]);
-              }
-            }
-          }
-        }
-      } else {
-        // larger batches (or int8 values): one value per chain step, one accumulator set
-#pragma unroll 2
-        for (int q = 0; q < iters; ++q) {
-          const int jl = msb32(lo), jh = msb32(hi);
-          lo = clear_bit(lo, jl);
-          hi = clear_bit(hi, jh);
-          uint16_t wl = 0, wh = 0;
-          if (ES == 2) {
-            if (jl >= 0) wl = reinterpret_cast<const uint16_t*>(vals)[top_lo - q];
-            if (jh >= 0) wh = reinterpret_cast<const uint16_t*>(vals)[top_hi - q];
-          } else {
-            if (jl >= 0) wl = i8_to_bf16(vals[top_lo - q]);
-            if (jh >= 0) wh = i8_to_bf16(vals[top_hi - q]);
-          }
-#pragma unroll
-          for (int r = 0; r < MP; ++r) {
-            const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
-            const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
-            if (jl >= 0) {
-              acc[2 * r] = fma_bf16(wl, lo16(xl), acc[2 * r]);
-              if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wl, hi16(xl), acc[2 * r + 1]);
-            }
-            if (jh >= 0) {
-              acc[2 * r] = fma_bf16(wh, lo16(xh), acc[2 * r]);
-              if (2 * r + 1 < M) acc[2 * r + 1] = fma_bf16(wh, hi16(xh), acc[2 * r + 1]);
-            }
-          }
-        }
-      }
-      if (ES == 2 && M <= 4) {
-#pragma unroll
-        for (int m = 0; m < (M <= 4 ? M : 1); ++m) acc[m] += accl[m] + acch[m];
-      }
+      uint32_t XL[(M + 1) / 2], XH[(M + 1) / 2];
+      load_x<M>(slot, p.chunk_region, lane, XL, XH);
+      row_dot<M, ES>(lo, hi, plo, pc, base + incl - pc, slot + kMaskBytes, XL, XH, acc);
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);
@@ -338,114 +466,151 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
       ++rb;
     }
     if (t_cur != T - 1 && w + 1 != w1) continue;
-    const int64_t seg_begin = rb_cur * T;
-    const int64_t n = rb_cur * kRows + tid;
-    const float sc = (ES == 1 && n < p.N) ? p.scale[n] : 1.f;
-    if constexpr (clustered) {
-      // Each CTA leaves its FP32 partial in its own shared memory; after a cluster barrier
-      // rank 0 adds the other ranks' partials in rank order (distributed shared memory)
-      // and writes y; a second barrier keeps every partial alive until then.
-      float* part = reinterpret_cast<float*>(smem + p.part_off);
-#pragma unroll
-      for (int m = 0; m < M; ++m) part[m * kRows + tid] = acc[m];
-      cluster_sync_all();
-      if (crank == 0) {
-        float sum[M];
-#pragma unroll
-        for (int m = 0; m < M; ++m) sum[m] = acc[m];
-        const uint32_t base = smem_u32(part) + 4u * (uint32_t)tid;
-        for (int r = 1; r < p.cluster; ++r) {
-          const uint32_t rb_addr = cluster_map(base, (uint32_t)r);
-          float v[M];
-#pragma unroll
-          for (int m = 0; m < M; ++m) v[m] = ld_cluster_f32(rb_addr + 4u * (uint32_t)(m * kRows));
-#pragma unroll
-          for (int m = 0; m < M; ++m) sum[m] += v[m];
-        }
-        if (n < p.N) {
-#pragma unroll
-          for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
-        }
-      }
-      cluster_sync_all();  // a clustered CTA covers one row block: this was its last chunk
-    } else {
-    if (seg_begin >= w0 && t_cur == T - 1) {
-      if (n < p.N) {
-#pragma unroll
-        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(acc[m] * sc);
-      }
-    } else {
-      const int my_slot = (rb_cur == rb_first) ? 0 : 1;
-      float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * (kRows * kMaxTokens);
-#pragma unroll
-      for (int m = 0; m < M; ++m) __stcg(wsp + m * kRows + tid, acc[m]);
-      __threadfence();
-      named_bar_sync(1, kConsumerWarps * 32);
-      const int64_t i_first = owner_of(seg_begin, p.W, p.G);
-      const int64_t i_last = owner_of(seg_begin + T - 1, p.W, p.G);
-      const int sf = (range_begin(i_first, p.W, p.G) / T == rb_cur) ? 0 : 1;
-      int* ctr = p.cnt + i_first * 2 + sf;
-      if (tid == 0) {
-        const int old = atomicAdd(ctr, 1);
-        *s_flag = (old == (int)(i_last - i_first)) ? 1 : 0;
-      }
-      named_bar_sync(1, kConsumerWarps * 32);
-      if (*s_flag) {
-        __threadfence();
-        float sum[M];
-#pragma unroll
-        for (int m = 0; m < M; ++m) sum[m] = 0.f;
-        // several contributors at a time: their loads are independent, the adds stay in
-        // CTA order
-        constexpr int kU = M <= 2 ? 8 : (M <= 8 ? 4 : 2);
-        for (int64_t i = i_first; i <= i_last; i += kU) {
-          float part[kU][M];
-#pragma unroll
-          for (int u = 0; u < kU; ++u) {
-            const int64_t ci = i + u;
-            if (ci <= i_last) {
-              const int sl = (range_begin(ci, p.W, p.G) / T == rb_cur) ? 0 : 1;
-              const float* src = p.ws + (ci * 2 + sl) * (kRows * kMaxTokens);
-#pragma unroll
-              for (int m = 0; m < M; ++m) part[u][m] = __ldcg(src + m * kRows + tid);
-            }
-          }
-#pragma unroll
-          for (int u = 0; u < kU; ++u)
-            if (i + u <= i_last) {
-#pragma unroll
-              for (int m = 0; m < M; ++m) sum[m] += part[u][m];
-            }
-        }
-        if (n < p.N) {
-#pragma unroll
-          for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
-        }
-        if (tid == 0) atomicExch(ctr, 0);
-      }
-      named_bar_sync(1, kConsumerWarps * 32);
-    }
-    }  // stream-K epilogue
+    row_block_end<M, ES, CL>(p, smem, s_flag, acc, rb_cur, rb_cur * T >= w0 && t_cur == T - 1,
+                             rb_cur == rb_first ? 0 : 1, crank, tid);
+    // (a clustered CTA covers one row block: this was its last item)
 #pragma unroll
     for (int m = 0; m < M; ++m) acc[m] = 0.f;
   }
 }
 
+// Warp-per-chunk kernel (M <= 4): consumer warp c takes items c, c + 4, c + 8, ... of
+// the CTA's range, and lane l owns rows 4l .. 4l+3 of its chunk, so one warp scan finds
+// every row's first value and each ring slot is released by the one warp that read it;
+// sixteen chunks per SM are in flight in the consumers instead of four.  At each row
+// block's end the four warps' partial sums meet in shared memory and are added in warp
+// order (deterministic) by thread r <-> row r, which runs the common epilogue.
+template <int M, int ES, bool CL>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const LinearParams p) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
+  uint64_t* empty = full + p.slots;
+  volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
+  float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [kConsumerWarps][M][kRows]
+  const int T = p.T;
+  const int slots = p.slots;  // >= kConsumerWarps
+  int64_t w0, w1;
+  uint32_t crank;
+  cta_range(p, CL, &w0, &w1, &crank);
+
+  if (tid == 0) {
+    for (int s = 0; s < slots; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    fence_barrier_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumerWarps) {
+    produce<M>(p, smem, full, empty, w0, w1, lane);
+    return;
+  }
+
+  pdl_wait();
+  pdl_launch_dependents();
+  bool dead = false;
+  int s = warp;  // ring slot of this warp's next item (item n uses slot n % slots)
+  uint32_t ph = 0;
+  int64_t w = w0 + warp;
+  const int64_t rb_first = w0 / T;
+  const int64_t rb_last = w1 > w0 ? (w1 - 1) / T : rb_first - 1;
+  for (int64_t rb = rb_first; rb <= rb_last; ++rb) {
+    const int64_t wb = rb * T > w0 ? rb * T : w0;
+    const int64_t we = (rb + 1) * T < w1 ? (rb + 1) * T : w1;
+    float acc[4][M];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int m = 0; m < M; ++m) acc[i][m] = 0.f;
+    for (; w < we; w += kConsumerWarps) {
+      if (!dead) {
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
+        if (!ok) {
+          dead = true;
+          set_status(p.status, kStatusTimeout);
+        }
+      }
+      if (!dead) {
+        const uint8_t* slot = smem + (size_t)s * p.slot_bytes;
+        // masks of rows 4l .. 4l+3: two 16-byte loads
+        const uint4 ma = *reinterpret_cast<const uint4*>(slot + 32 * lane);
+        const uint4 mb = *reinterpret_cast<const uint4*>(slot + 32 * lane + 16);
+        const uint32_t lo[4] = {ma.x, ma.z, mb.x, mb.z}, hi[4] = {ma.y, ma.w, mb.y, mb.w};
+        int plo[4], pc[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          plo[i] = __popc(lo[i]);
+          pc[i] = plo[i] + __popc(hi[i]);
+        }
+        const int tot = pc[0] + pc[1] + pc[2] + pc[3];
+        int incl = tot;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+          const int u = __shfl_up_sync(0xffffffffu, incl, d);
+          if (lane >= d) incl += u;
+        }
+        int e = incl - tot;  // first value of row 4l
+        uint32_t XL[(M + 1) / 2], XH[(M + 1) / 2];
+        load_x<M>(slot, p.chunk_region, lane, XL, XH);
+        const uint8_t* vals = slot + kMaskBytes;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          row_dot<M, ES>(lo[i], hi[i], plo[i], pc[i], e, vals, XL, XH, acc[i]);
+          e += pc[i];
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[s]);
+      if ((s += kConsumerWarps) >= slots) {
+        s -= slots;
+        ph ^= 1u;
+      }
+    }
+    // the four warps' partials for rows 4l + i, added in warp order by thread r <-> row r
+#pragma unroll
+    for (int m = 0; m < M; ++m)
+      *reinterpret_cast<float4*>(comb + (warp * M + m) * kRows + 4 * lane) =
+          make_float4(acc[0][m], acc[1][m], acc[2][m], acc[3][m]);
+    named_bar_sync(2, kConsumerWarps * 32);
+    float sum[M];
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      sum[m] = comb[m * kRows + tid];
+#pragma unroll
+      for (int c = 1; c < kConsumerWarps; ++c) sum[m] += comb[(c * M + m) * kRows + tid];
+    }
+    named_bar_sync(2, kConsumerWarps * 32);  // comb is rewritten at the next row block
+    row_block_end<M, ES, CL>(p, smem, s_flag, sum, rb, wb == rb * T && we == (rb + 1) * T,
+                             rb == rb_first ? 0 : 1, crank, tid);
+  }
+}
+
+// kind 0: thread-per-row kernel; kind 1: warp-per-chunk kernel (M <= 4)
 template <int M, int ES>
-sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem) {
-  auto kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
-  static bool configured[2][kMaxDevices] = {};  // kernel attributes, once per device
+sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind) {
+  void (*kern)(const LinearParams);
+  if constexpr (M <= 4) {
+    if (kind == 1)
+      kern = p.cluster > 1 ? linear_ccw_kernel<M, ES, true> : linear_ccw_kernel<M, ES, false>;
+    else
+      kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
+  } else {
+    kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
+  }
+  static bool configured[2][2][kMaxDevices] = {};  // kernel attributes, once per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
   const int ci = p.cluster > 1 ? 1 : 0;
-  if (!configured[ci][dev]) {
+  if (!configured[kind][ci][dev]) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess ||
         (ci && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
       cudaGetLastError();
       return SP_ERR_CUDA;
     }
-    configured[ci][dev] = true;
+    configured[kind][ci][dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)p.G);
@@ -473,24 +638,24 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem) {
 }
 
 template <int ES>
-sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem) {
+sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, int kind) {
   switch (p.M) {
-    case 1: return launch_one<1, ES>(p, stream, smem);
-    case 2: return launch_one<2, ES>(p, stream, smem);
-    case 3: return launch_one<3, ES>(p, stream, smem);
-    case 4: return launch_one<4, ES>(p, stream, smem);
-    case 5: return launch_one<5, ES>(p, stream, smem);
-    case 6: return launch_one<6, ES>(p, stream, smem);
-    case 7: return launch_one<7, ES>(p, stream, smem);
-    case 8: return launch_one<8, ES>(p, stream, smem);
-    case 9: return launch_one<9, ES>(p, stream, smem);
-    case 10: return launch_one<10, ES>(p, stream, smem);
-    case 11: return launch_one<11, ES>(p, stream, smem);
-    case 12: return launch_one<12, ES>(p, stream, smem);
-    case 13: return launch_one<13, ES>(p, stream, smem);
-    case 14: return launch_one<14, ES>(p, stream, smem);
-    case 15: return launch_one<15, ES>(p, stream, smem);
-    case 16: return launch_one<16, ES>(p, stream, smem);
+    case 1: return launch_one<1, ES>(p, stream, smem, kind);
+    case 2: return launch_one<2, ES>(p, stream, smem, kind);
+    case 3: return launch_one<3, ES>(p, stream, smem, kind);
+    case 4: return launch_one<4, ES>(p, stream, smem, kind);
+    case 5: return launch_one<5, ES>(p, stream, smem, kind);
+    case 6: return launch_one<6, ES>(p, stream, smem, kind);
+    case 7: return launch_one<7, ES>(p, stream, smem, kind);
+    case 8: return launch_one<8, ES>(p, stream, smem, kind);
+    case 9: return launch_one<9, ES>(p, stream, smem, kind);
+    case 10: return launch_one<10, ES>(p, stream, smem, kind);
+    case 11: return launch_one<11, ES>(p, stream, smem, kind);
+    case 12: return launch_one<12, ES>(p, stream, smem, kind);
+    case 13: return launch_one<13, ES>(p, stream, smem, kind);
+    case 14: return launch_one<14, ES>(p, stream, smem, kind);
+    case 15: return launch_one<15, ES>(p, stream, smem, kind);
+    case 16: return launch_one<16, ES>(p, stream, smem, kind);
     default: return SP_ERR_INVALID_ARG;
   }
 }
@@ -553,14 +718,24 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.x = x + m0 * h->K;
     p.y = y + m0 * h->N;
     p.slot_bytes = p.chunk_region + (uint32_t)Mt * 128u;
-    // slots, 2*slots mbarriers (<= 256 B), the flag and (cluster mode) the FP32 partial
+    // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag, the warps'
+    // partials (warp-per-chunk kernel) and the CTA's FP32 partial (cluster mode)
     const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
-    int slots = (int)std::min<size_t>(16, (kSmemBudget - 256 - 16 - part_bytes) / p.slot_bytes);
+    const size_t comb_bytes = (size_t)kConsumerWarps * kRows * Mt * sizeof(float);
+    int kind = 0;
+    size_t ring = kSmemBudget - 256 - 16 - part_bytes;
+    if (Mt <= 4 && (ring - comb_bytes) / p.slot_bytes >= (size_t)kConsumerWarps) {
+      kind = 1;
+      ring -= comb_bytes;
+    }
+    const int slots = (int)std::min<size_t>(16, ring / p.slot_bytes);
     if (slots < 2) return SP_ERR_UNSUPPORTED;
     p.slots = slots;
-    p.part_off = (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 15) / 16 * 16);
+    p.comb_off = (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 15) / 16 * 16);
+    p.part_off = p.comb_off + (uint32_t)(kind == 1 ? comb_bytes : 0);
     const size_t smem = p.part_off + part_bytes;
-    const sp_status st = h->esize == 2 ? dispatch_m<2>(p, stream, smem) : dispatch_m<1>(p, stream, smem);
+    const sp_status st =
+        h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind) : dispatch_m<1>(p, stream, smem, kind);
     if (st != SP_OK) return st;
   }
   return SP_OK;
