@@ -120,9 +120,11 @@ __device__ __forceinline__ void cta_range(const LinearParams& p, bool clustered,
 // warp walks the chunk list (it shares the offset window); lane 0 issues.  Weight bytes
 // do not depend on the previous kernel in the stream: the first ring fill is issued
 // before griddepcontrol.wait; every x copy comes after it.
+// tag[s] = n records that slot s has been claimed for item n (written once the slot's
+// previous item has been consumed), for consumers that do not read every item.
 template <int M>
 __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, uint64_t* full, uint64_t* empty,
-                                        int64_t w0, int64_t w1, int lane) {
+                                        volatile int* tag, int64_t w0, int64_t w1, int lane) {
   const int T = p.T;
   const int slots = p.slots;
   const uint64_t pol = policy_evict_first();
@@ -137,6 +139,7 @@ __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, ui
       if (lane == 0) {
         const uint32_t bytes = (uint32_t)(o1 - o0);
         const int valid = (int)imin64((int64_t)kTileK, p.K - (int64_t)kTileK * t);
+        tag[i] = (int)i;
         mbar_arrive_expect_tx(&full[i], bytes + (uint32_t)M * (uint32_t)valid * 2u);
         bulk_g2s_hint(smem + (size_t)i * p.slot_bytes, p.buf + o0, bytes, &full[i], pol);
       }
@@ -163,6 +166,7 @@ __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, ui
           failed = true;
         } else {
           const uint32_t bytes = (uint32_t)(o1 - o0);
+          tag[s] = (int)n_issued;
           mbar_arrive_expect_tx(&full[s], bytes + (uint32_t)M * xb);
           bulk_g2s_hint(slot, p.buf + o0, bytes, &full[s], pol);
         }
@@ -393,6 +397,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
   uint64_t* empty = full + p.slots;
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
+  volatile int* tag = s_flag + 4;
   const int T = p.T;
   const int slots = p.slots;
   int64_t w0, w1;
@@ -403,13 +408,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
     for (int s = 0; s < slots; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kConsumerWarps);
+      tag[s] = -1;
     }
     fence_barrier_init();
   }
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    produce<M>(p, smem, full, empty, w0, w1, lane);
+    produce<M>(p, smem, full, empty, tag, w0, w1, lane);
     return;
   }
 
@@ -487,6 +493,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
   uint64_t* empty = full + p.slots;
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
+  volatile int* tag = s_flag + 4;
   float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [kConsumerWarps][M][kRows]
   const int T = p.T;
   const int slots = p.slots;  // >= kConsumerWarps
@@ -498,13 +505,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
     for (int s = 0; s < slots; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
+      tag[s] = -1;
     }
     fence_barrier_init();
   }
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    produce<M>(p, smem, full, empty, w0, w1, lane);
+    produce<M>(p, smem, full, empty, tag, w0, w1, lane);
     return;
   }
 
@@ -525,6 +533,21 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
 #pragma unroll
       for (int m = 0; m < M; ++m) acc[i][m] = 0.f;
     for (; w < we; w += kConsumerWarps) {
+      if (!dead && tag[s] != (int)(w - w0)) {
+        // the slot may still hold an earlier item of another warp: wait until the producer
+        // has claimed it for this one (it does so only once that item was consumed), so
+        // the parity wait below cannot match an older phase of the slot's barrier
+        const uint64_t t0 = global_ns();
+        while (tag[s] != (int)(w - w0)) {
+          __nanosleep(32);
+          if (global_ns() - t0 > p.timeout_ns) {
+            dead = true;
+            set_status(p.status, kStatusTimeout);
+            break;
+          }
+        }
+        dead = __any_sync(0xffffffffu, dead);
+      }
       if (!dead) {
         const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
         if (!ok) {
@@ -718,12 +741,13 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.x = x + m0 * h->K;
     p.y = y + m0 * h->N;
     p.slot_bytes = p.chunk_region + (uint32_t)Mt * 128u;
-    // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag, the warps'
-    // partials (warp-per-chunk kernel) and the CTA's FP32 partial (cluster mode)
+    // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag (16 B), the slot
+    // tags (<= 64 B), the warps' partials (warp-per-chunk kernel) and the CTA's FP32
+    // partial (cluster mode)
     const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
     const size_t comb_bytes = (size_t)kConsumerWarps * kRows * Mt * sizeof(float);
     int kind = 0;
-    size_t ring = kSmemBudget - 256 - 16 - part_bytes;
+    size_t ring = kSmemBudget - 256 - 16 - 64 - part_bytes;
     if (Mt <= 4 && (ring - comb_bytes) / p.slot_bytes >= (size_t)kConsumerWarps) {
       kind = 1;
       ring -= comb_bytes;
@@ -731,7 +755,8 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     const int slots = (int)std::min<size_t>(16, ring / p.slot_bytes);
     if (slots < 2) return SP_ERR_UNSUPPORTED;
     p.slots = slots;
-    p.comb_off = (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 15) / 16 * 16);
+    p.comb_off =
+        (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 4 * (size_t)slots + 15) / 16 * 16);
     p.part_off = p.comb_off + (uint32_t)(kind == 1 ? comb_bytes : 0);
     const size_t smem = p.part_off + part_bytes;
     const sp_status st =

@@ -657,7 +657,10 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   // base alignment + barriers (2 per slot, 2 per A stage, 2 for D), TMEM address, flag
   const size_t tail =
       1024 + 8 * (2 * kMaxSlots + 2 * kMaxAStages + kMaxDBufs * (kExpGroups + 1)) + 4 + 4 * kExpGroups + 16;
-  const int slots = (int)std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes);
+  // an even number of slots: the expander warpgroups take alternate items, so a slot's
+  // previous item then belongs to the warpgroup now waiting on it, which keeps the parity
+  // wait on the slot's full barrier exact
+  const int slots = (int)std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes) & ~1;
   if (slots < 2) return SP_ERR_UNSUPPORTED;
   p.slots = slots;
   // at least 116 KB so that two CTAs never share an SM (each allocates 512 TMEM columns)
