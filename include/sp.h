@@ -63,7 +63,9 @@ typedef enum sp_status {
 
 typedef enum sp_dtype { SP_BF16 = 0, SP_INT8 = 1 } sp_dtype;
 
-/* Kernel family used by sp_linear_ex.  SP_PATH_AUTO picks by batch size M. */
+/* Kernel family used by sp_linear_ex.  SP_PATH_AUTO picks by batch size M: the CUDA-core
+   family for M <= 10 (bf16 values) or M <= 13 (int8 values), the tensor-core family above
+   (the measured crossover on the Llama-2-7B shapes). */
 typedef enum sp_path {
   SP_PATH_AUTO = 0,
   SP_PATH_CUDA_CORE = 1,    /* popc-prefix expansion, FP32 FMA on CUDA cores */
@@ -124,6 +126,22 @@ sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_de
 /* sp_linear with an explicit kernel family (tests run each family on its own). */
 sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
                        size_t workspace_bytes, sp_path path, void* stream);
+
+/* Kernels that sp_linear_ex can launch (reported by sp_launch_count). */
+enum {
+  SP_KERNEL_NONE = 0,
+  SP_KERNEL_CC_THREAD_PER_ROW = 1,  /* linear_cc_kernel: four warps share a chunk, thread = row */
+  SP_KERNEL_CC_WARP_PER_CHUNK = 2,  /* linear_ccw_kernel (M <= 4): a warp per chunk, lane = 4 rows */
+  SP_KERNEL_TENSOR_CORE = 3         /* linear_tc_kernel */
+};
+
+/* Number of kernel launches that sp_linear_ex(h, x, m, y, ws, ws_bytes, path, stream)
+ * makes, written to *launches: 0 for m == 0, one per 16 batch rows on the CUDA-core
+ * family, one on the tensor-core family; if `kernel` is not null, the SP_KERNEL_* value
+ * of the kernel used for the first 16 rows (or all rows) goes there.  For callers that
+ * count launches or label profiles.  Host only: no GPU work.  SP_ERR_BAD_HANDLE for a
+ * dead handle, SP_ERR_INVALID_ARG for m < 0, an unknown path or a null `launches`. */
+sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* launches, int32_t* kernel);
 
 /* sp_linear for callers that may not allocate device memory (the paper has no
  * counterpart; this is a deployment convenience).  Some callers receive only their

@@ -22,8 +22,17 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 bool live(const sp_matrix* h) { return h && h->magic == SP_MAGIC; }
 
 // Largest batch that the CUDA-core family takes under SP_PATH_AUTO; larger batches go
-// to the tensor-core family.
-constexpr int64_t kCudaCoreMaxM = 16;
+// to the tensor-core family.  Measured crossover on the Llama-2-7B shapes at 70%: the
+// CUDA-core path costs ~M FMAs per kept weight and the tensor-core path a fixed
+// expansion per chunk, so the tensor cores win from M ~ 11 (bf16 values) and from
+// M ~ 14 (int8 values, whose CUDA-core loop is cheaper and whose expansion costs more).
+constexpr int64_t kCudaCoreMaxM_bf16 = 10;
+constexpr int64_t kCudaCoreMaxM_int8 = 13;
+
+bool uses_tensor_cores(const sp_matrix* h, int64_t m, sp_path path) {
+  const int64_t cc_max = h->esize == 1 ? kCudaCoreMaxM_int8 : kCudaCoreMaxM_bf16;
+  return path == SP_PATH_TENSOR_CORE || (path == SP_PATH_AUTO && m > cc_max);
+}
 }  // namespace
 
 int* device_status_ptr() {
@@ -120,11 +129,28 @@ sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y
   // The documented contract, whatever kernel runs: a workspace of sp_workspace_size bytes.
   if (!workspace_dev || workspace_bytes < std::max(workspace_bytes_cc(h, m), workspace_bytes_tc(h, m)))
     return SP_ERR_WORKSPACE;
-  if (path == SP_PATH_TENSOR_CORE || (path == SP_PATH_AUTO && m > kCudaCoreMaxM))
+  if (uses_tensor_cores(h, m, path))
     return launch_linear_tc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
                             workspace_bytes, (cudaStream_t)stream);
   return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
                           workspace_bytes, (cudaStream_t)stream);
+}
+
+sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* launches, int32_t* kernel) {
+  if (!h || h->magic != SP_MAGIC) return SP_ERR_BAD_HANDLE;
+  if (m < 0 || !launches || (path != SP_PATH_AUTO && path != SP_PATH_CUDA_CORE && path != SP_PATH_TENSOR_CORE))
+    return SP_ERR_INVALID_ARG;
+  const bool tc = uses_tensor_cores(h, m, path);
+  *launches = m == 0 ? 0 : tc ? 1 : (m + kMaxTokens - 1) / kMaxTokens;
+  if (kernel) {
+    if (m == 0)
+      *kernel = SP_KERNEL_NONE;
+    else if (tc)
+      *kernel = SP_KERNEL_TENSOR_CORE;
+    else
+      *kernel = cc_kernel_kind(h, m) == 1 ? SP_KERNEL_CC_WARP_PER_CHUNK : SP_KERNEL_CC_THREAD_PER_ROW;
+  }
+  return SP_OK;
 }
 
 sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,

@@ -74,6 +74,7 @@ struct LinearParams {
 // [arrival counters for up to 2 * kMaxGridPerSm * SMs partial slots][fp32 partials].
 // Every call leaves the counters at zero.
 constexpr int kMaxGridPerSm = 4;
+constexpr int kMaxTokens = 16;  // batch rows per CUDA-core launch (larger batches take several)
 inline size_t ws_counter_bytes(int num_sms) {
   return ((size_t)2 * kMaxGridPerSm * num_sms * sizeof(int) + 255) / 256 * 256;
 }
@@ -227,6 +228,7 @@ sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream, bool allow_cluster = true);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
+int cc_kernel_kind(const sp_matrix* h, int64_t M);  // 0 thread-per-row, 1 warp-per-chunk, -1 none fits
 sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream);
 size_t workspace_bytes_tc(const sp_matrix* h, int64_t M);

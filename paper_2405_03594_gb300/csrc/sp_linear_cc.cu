@@ -30,7 +30,6 @@ namespace {
 
 constexpr int kConsumerWarps = 4;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;
-constexpr int kMaxTokens = 16;  // batch rows per launch of this kernel
 constexpr int kMaxDevices = 64;
 constexpr int kCtasPerSm = 4;
 constexpr size_t kSmemBudget = 53 * 1024;  // ring slots per CTA; four CTAs share one SM
@@ -707,7 +706,44 @@ int grid_cc(const sp_matrix* h) {
   return (int)std::min<int64_t>(per_sm * h->num_sms, W);
 }
 
+// Shared-memory plan of one launch with Mt batch rows: ring slots, whether the
+// warp-per-chunk kernel runs (M <= 4 and room for a slot per consumer warp after its
+// partials), and the offsets of the warps' partials and of the cluster partial.
+struct CcPlan {
+  int slots, kind;
+  uint32_t slot_bytes, comb_off, part_off;
+  size_t smem;
+};
+bool cc_plan(const sp_matrix* h, int Mt, int S, CcPlan* pl) {
+  const uint32_t chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
+  pl->slot_bytes = chunk_region + (uint32_t)Mt * 128u;
+  // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag (16 B), the slot
+  // tags (<= 64 B), the warps' partials (warp-per-chunk kernel) and the CTA's FP32
+  // partial (cluster mode)
+  const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
+  const size_t comb_bytes = (size_t)kConsumerWarps * kRows * Mt * sizeof(float);
+  pl->kind = 0;
+  size_t ring = kSmemBudget - 256 - 16 - 64 - part_bytes;
+  if (Mt <= 4 && (ring - comb_bytes) / pl->slot_bytes >= (size_t)kConsumerWarps) {
+    pl->kind = 1;
+    ring -= comb_bytes;
+  }
+  pl->slots = (int)std::min<size_t>(16, ring / pl->slot_bytes);
+  if (pl->slots < 2) return false;
+  pl->comb_off = (uint32_t)(((size_t)pl->slots * pl->slot_bytes + 2 * (size_t)pl->slots * 8 + 16 +
+                             4 * (size_t)pl->slots + 15) /
+                            16 * 16);
+  pl->part_off = pl->comb_off + (uint32_t)(pl->kind == 1 ? comb_bytes : 0);
+  pl->smem = pl->part_off + part_bytes;
+  return true;
+}
+
 }  // namespace
+
+int cc_kernel_kind(const sp_matrix* h, int64_t M) {
+  CcPlan pl;
+  return cc_plan(h, (int)std::min<int64_t>(kMaxTokens, M), cluster_cc(h), &pl) ? pl.kind : -1;
+}
 
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
   const size_t G = (size_t)grid_cc(h);
@@ -740,25 +776,14 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.M = Mt;
     p.x = x + m0 * h->K;
     p.y = y + m0 * h->N;
-    p.slot_bytes = p.chunk_region + (uint32_t)Mt * 128u;
-    // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag (16 B), the slot
-    // tags (<= 64 B), the warps' partials (warp-per-chunk kernel) and the CTA's FP32
-    // partial (cluster mode)
-    const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
-    const size_t comb_bytes = (size_t)kConsumerWarps * kRows * Mt * sizeof(float);
-    int kind = 0;
-    size_t ring = kSmemBudget - 256 - 16 - 64 - part_bytes;
-    if (Mt <= 4 && (ring - comb_bytes) / p.slot_bytes >= (size_t)kConsumerWarps) {
-      kind = 1;
-      ring -= comb_bytes;
-    }
-    const int slots = (int)std::min<size_t>(16, ring / p.slot_bytes);
-    if (slots < 2) return SP_ERR_UNSUPPORTED;
-    p.slots = slots;
-    p.comb_off =
-        (uint32_t)(((size_t)slots * p.slot_bytes + 2 * (size_t)slots * 8 + 16 + 4 * (size_t)slots + 15) / 16 * 16);
-    p.part_off = p.comb_off + (uint32_t)(kind == 1 ? comb_bytes : 0);
-    const size_t smem = p.part_off + part_bytes;
+    CcPlan pl;
+    if (!cc_plan(h, Mt, S, &pl)) return SP_ERR_UNSUPPORTED;
+    p.slot_bytes = pl.slot_bytes;
+    p.slots = pl.slots;
+    p.comb_off = pl.comb_off;
+    p.part_off = pl.part_off;
+    const int kind = pl.kind;
+    const size_t smem = pl.smem;
     const sp_status st =
         h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind) : dispatch_m<1>(p, stream, smem, kind);
     if (st != SP_OK) return st;

@@ -24,9 +24,13 @@ STATUS = {
     5: "SP_ERR_OUT_OF_MEMORY", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_BAD_HANDLE", 8: "SP_ERR_WORKSPACE",
 }
 # every function declared in include/sp.h and include/sp_stack.h
-EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_linear_noalloc",
+EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
+           "sp_linear_noalloc",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
            "sp_copy_columns", "sp_residual_add", "sp_mul_halves"]
+
+
+KERNELS = {0: "", 1: "linear_cc_kernel", 2: "linear_ccw_kernel", 3: "linear_tc_kernel"}  # SP_KERNEL_*
 
 
 class SpError(RuntimeError):
@@ -133,6 +137,18 @@ class SparseMatrix:
         b = ctypes.c_size_t()
         _check(_lib.sp_workspace_size(self._h, m, ctypes.byref(b)), "sp_workspace_size")
         return int(b.value)
+
+    def launch_count(self, m: int, path: str = "auto") -> int:
+        """Kernel launches that linear() makes for a batch of m rows on `path`."""
+        n = ctypes.c_int64()
+        _check(_lib.sp_launch_count(self._h, m, PATHS[path], ctypes.byref(n), None), "sp_launch_count")
+        return int(n.value)
+
+    def kernel_name(self, m: int, path: str = "auto") -> str:
+        """Name of the kernel that linear() runs for a batch of m rows on `path`."""
+        n, k = ctypes.c_int64(), ctypes.c_int32()
+        _check(_lib.sp_launch_count(self._h, m, PATHS[path], ctypes.byref(n), ctypes.byref(k)), "sp_launch_count")
+        return KERNELS[k.value]
 
     def linear(self, x: torch.Tensor, out: torch.Tensor | None = None, workspace: torch.Tensor | None = None,
                path: str = "auto", stream=None) -> torch.Tensor:

@@ -84,10 +84,10 @@ class LinearStack:
                                  for n in SHAPES)
 
     def launches_per_step(self, M: int, reset: bool = True) -> int:
-        """libsp kernels per step: four sparse linears and four glue kernels per layer
-        (the CUDA-core family takes at most 16 batch rows per launch), plus the input copy."""
-        per_linear = (M + 15) // 16 if self.path == "cuda_core" else 1
-        return self.layers * (4 * per_linear + 4) + (1 if reset else 0)
+        """libsp kernels per step: the four sparse linears (as many launches as the library
+        reports for M rows) and four glue kernels per layer, plus the input copy."""
+        per_layer = sum(self.mats[n][0].launch_count(M, self.path) for n in SHAPES)
+        return self.layers * (per_layer + 4) + (1 if reset else 0)
 
     def set_input(self, x: torch.Tensor):
         """Token embeddings [M, 4096] bf16 for the next steps."""

@@ -221,6 +221,25 @@ def test_tensor_core_short_segments(sp, oracle, N, K, M):
     gu.assert_close(gu.bf16_from_dev(y), _ref(oracle, vals, s, mask, x), f"{N}x{K} M={M}")
 
 
+def test_launch_count(sp):
+    """sp_launch_count: one launch per 16 rows on the CUDA-core family, one on the tensor-core
+    family, and AUTO switches at M = 11 for bf16 values and at M = 14 for int8 values."""
+    vals, s, mask, _ = _case(300, 200, 1, 70, seed=5)
+    h = sp.compress(gu.bf16_to_dev(vals), gu.u8_to_dev(mask))
+    q, sc = __import__("paper_2405_03594_gb300").synth.quantize_int8(vals, mask)
+    h8 = sp.compress(gu.i8_to_dev(q), gu.u8_to_dev(mask), gu.f32_to_dev(sc))
+    assert h.launch_count(0) == 0
+    assert [h.launch_count(m, "cuda_core") for m in (1, 16, 17, 40)] == [1, 1, 2, 3]
+    assert [h.launch_count(m, "tensor_core") for m in (1, 16, 17, 300)] == [1, 1, 1, 1]
+    assert [h.launch_count(m) for m in (1, 10, 11, 40)] == [1, 1, 1, 1]
+    assert [h8.launch_count(m) for m in (13, 14, 17)] == [1, 1, 1]
+    assert h8.launch_count(40, "cuda_core") == 3
+    with pytest.raises(sp.SpError):
+        h.launch_count(-1)
+    assert h.kernel_name(1) == "linear_ccw_kernel" and h.kernel_name(8) == "linear_cc_kernel"
+    assert h.kernel_name(11) == "linear_tc_kernel" and h.kernel_name(3, "tensor_core") == "linear_tc_kernel"
+
+
 def test_shared_workspace_across_grids(sp, oracle):
     """Matrices whose launches use different grid sizes share one workspace, interleaved:
     the split-K counters must never be overlaid by another call's partials."""
