@@ -479,12 +479,163 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
   }
 }
 
+// ---------------------------------------------------------------- asynchronous row-block end
+// (warp-per-chunk kernel, stream-K): each warp flushes its partials into a double-buffered
+// combine area and the last of the four to flush adds them and runs the epilogue alone
+// while the others go on with the next row block.
+struct FlushCtl {
+  int flushed[2];  // warps that have flushed the row block held by buffer b
+  int ready[2];    // local row block that may be written into buffer b next
+};
+
+// Rows 4*lane + i of row block rb: y = bf16(s * scale)
+template <int M, int ES>
+__device__ __forceinline__ void store_rows(const LinearParams& p, const float (&s)[4][M], int64_t rb, int lane) {
+  const int64_t n0 = rb * kRows + 4 * lane;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t n = n0 + i;
+    if (n < p.N) {
+      const float sc = ES == 1 ? p.scale[n] : 1.f;
+#pragma unroll
+      for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(s[i][m] * sc);
+    }
+  }
+}
+
+// End of row block rb run by one warp (rows 4*lane + i): a CTA that covered the whole row
+// block writes y; otherwise it stores its partial in workspace slot `my_slot` and the last
+// of the row block's CTAs to arrive adds the partials in CTA order and writes y.
+template <int M, int ES>
+__device__ __forceinline__ void row_block_end_warp(const LinearParams& p, const float (&sum)[4][M], int64_t rb,
+                                                   bool complete, int my_slot, int lane) {
+  if (complete) {
+    store_rows<M, ES>(p, sum, rb, lane);
+    return;
+  }
+  const int T = p.T;
+  float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * (kRows * kMaxTokens) + 4 * lane;
+#pragma unroll
+  for (int m = 0; m < M; ++m)
+    __stcg(reinterpret_cast<float4*>(wsp + m * kRows), make_float4(sum[0][m], sum[1][m], sum[2][m], sum[3][m]));
+  __threadfence();
+  __syncwarp();
+  const int64_t seg_begin = rb * T;
+  const int64_t i_first = owner_of(seg_begin, p.W, p.G);
+  const int64_t i_last = owner_of(seg_begin + T - 1, p.W, p.G);
+  const int sf = (range_begin(i_first, p.W, p.G) / T == rb) ? 0 : 1;
+  int* ctr = p.cnt + i_first * 2 + sf;
+  int last = 0;
+  if (lane == 0) last = (atomicAdd(ctr, 1) == (int)(i_last - i_first)) ? 1 : 0;
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence();
+  float tot[4][M];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int m = 0; m < M; ++m) tot[i][m] = 0.f;
+  // several contributors at a time: their loads are independent, the adds stay in CTA order
+  constexpr int kU = M <= 2 ? 4 : 1;
+  for (int64_t i = i_first; i <= i_last; i += kU) {
+    float4 part[kU][M];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t ci = i + u;
+      if (ci <= i_last) {
+        const int sl = (range_begin(ci, p.W, p.G) / T == rb) ? 0 : 1;
+        const float* src = p.ws + (ci * 2 + sl) * (kRows * kMaxTokens) + 4 * lane;
+#pragma unroll
+        for (int m = 0; m < M; ++m) part[u][m] = __ldcg(reinterpret_cast<const float4*>(src + m * kRows));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u)
+      if (i + u <= i_last) {
+#pragma unroll
+        for (int m = 0; m < M; ++m) {
+          tot[0][m] += part[u][m].x;
+          tot[1][m] += part[u][m].y;
+          tot[2][m] += part[u][m].z;
+          tot[3][m] += part[u][m].w;
+        }
+      }
+  }
+  store_rows<M, ES>(p, tot, rb, lane);
+  if (lane == 0) atomicExch(ctr, 0);
+}
+
+// Warp `warp` is done with local row block k of its CTA: its partial sums go to buffer
+// k % 2, and the last of the kConsumerWarps warps to flush k adds them in warp order and
+// runs the row block's end.
+template <int M, int ES>
+__device__ __forceinline__ void flush_async(const LinearParams& p, FlushCtl* ctl, float* comb,
+                                            const float (&acc)[4][M], int k, int64_t rb_first, int64_t w0,
+                                            int64_t w1, int warp, int lane) {
+  const int T = p.T;
+  const int b = k & 1;
+  volatile int* ready = ctl->ready;
+  if (ready[b] != k) {
+    // the buffer still holds row block k - 2, whose end is under way
+    const uint64_t t0 = global_ns();
+    while (ready[b] != k) {
+      __nanosleep(64);
+      if (global_ns() - t0 > p.timeout_ns) {
+        set_status(p.status, kStatusTimeout);
+        break;
+      }
+    }
+  }
+  float* cb = comb + (size_t)b * kConsumerWarps * M * kRows;
+#pragma unroll
+  for (int m = 0; m < M; ++m)
+    *reinterpret_cast<float4*>(cb + (warp * M + m) * kRows + 4 * lane) =
+        make_float4(acc[0][m], acc[1][m], acc[2][m], acc[3][m]);
+  __syncwarp();
+  int last = 0;
+  if (lane == 0) {
+    __threadfence_block();
+    last = (atomicAdd(&ctl->flushed[b], 1) == kConsumerWarps - 1) ? 1 : 0;
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence_block();
+  float sum[4][M];
+#pragma unroll
+  for (int m = 0; m < M; ++m) {
+    float4 a = *reinterpret_cast<const float4*>(cb + m * kRows + 4 * lane);
+#pragma unroll
+    for (int c = 1; c < kConsumerWarps; ++c) {
+      const float4 v = *reinterpret_cast<const float4*>(cb + (c * M + m) * kRows + 4 * lane);
+      a.x += v.x;
+      a.y += v.y;
+      a.z += v.z;
+      a.w += v.w;
+    }
+    sum[0][m] = a.x;
+    sum[1][m] = a.y;
+    sum[2][m] = a.z;
+    sum[3][m] = a.w;
+  }
+  __syncwarp();
+  if (lane == 0) ctl->flushed[b] = 0;
+  const int64_t rb = rb_first + k;
+  row_block_end_warp<M, ES>(p, sum, rb, rb * T >= w0 && (rb + 1) * T <= w1, k == 0 ? 0 : 1, lane);
+  __syncwarp();
+  if (lane == 0) {
+    __threadfence_block();
+    ready[b] = k + 2;
+  }
+}
+
 // Warp-per-chunk kernel (M <= 4): consumer warp c takes items c, c + 4, c + 8, ... of
 // the CTA's range, and lane l owns rows 4l .. 4l+3 of its chunk, so one warp scan finds
 // every row's first value and each ring slot is released by the one warp that read it;
 // sixteen chunks per SM are in flight in the consumers instead of four.  At each row
 // block's end the four warps' partial sums meet in shared memory and are added in warp
-// order (deterministic) by thread r <-> row r, which runs the common epilogue.
+// order (deterministic): in stream-K mode by the last warp to get there, which runs the
+// row block's end alone while the others go on (flush_async); in cluster mode, where a
+// CTA's one row block ends with its range, by thread r <-> row r after a barrier.
 template <int M, int ES, bool CL>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -493,7 +644,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
   uint64_t* empty = full + p.slots;
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
   volatile int* tag = s_flag + 4;
-  float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [kConsumerWarps][M][kRows]
+  float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [2][kConsumerWarps][M][kRows]
+  FlushCtl* fctl = reinterpret_cast<FlushCtl*>(comb + 2 * kConsumerWarps * M * kRows);
   const int T = p.T;
   const int slots = p.slots;  // >= kConsumerWarps
   int64_t w0, w1;
@@ -505,6 +657,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
       tag[s] = -1;
+    }
+    for (int b = 0; b < 2; ++b) {
+      fctl->flushed[b] = 0;
+      fctl->ready[b] = b;
     }
     fence_barrier_init();
   }
@@ -590,22 +746,26 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
         ph ^= 1u;
       }
     }
-    // the four warps' partials for rows 4l + i, added in warp order by thread r <-> row r
+    if constexpr (!CL) {
+      flush_async<M, ES>(p, fctl, comb, acc, (int)(rb - rb_first), rb_first, w0, w1, warp, lane);
+    } else {
+      // the four warps' partials for rows 4l + i, added in warp order by thread r <-> row r
 #pragma unroll
-    for (int m = 0; m < M; ++m)
-      *reinterpret_cast<float4*>(comb + (warp * M + m) * kRows + 4 * lane) =
-          make_float4(acc[0][m], acc[1][m], acc[2][m], acc[3][m]);
-    named_bar_sync(2, kConsumerWarps * 32);
-    float sum[M];
+      for (int m = 0; m < M; ++m)
+        *reinterpret_cast<float4*>(comb + (warp * M + m) * kRows + 4 * lane) =
+            make_float4(acc[0][m], acc[1][m], acc[2][m], acc[3][m]);
+      named_bar_sync(2, kConsumerWarps * 32);
+      float sum[M];
 #pragma unroll
-    for (int m = 0; m < M; ++m) {
-      sum[m] = comb[m * kRows + tid];
+      for (int m = 0; m < M; ++m) {
+        sum[m] = comb[m * kRows + tid];
 #pragma unroll
-      for (int c = 1; c < kConsumerWarps; ++c) sum[m] += comb[(c * M + m) * kRows + tid];
+        for (int c = 1; c < kConsumerWarps; ++c) sum[m] += comb[(c * M + m) * kRows + tid];
+      }
+      named_bar_sync(2, kConsumerWarps * 32);  // comb is rewritten at the next row block
+      row_block_end<M, ES, CL>(p, smem, s_flag, sum, rb, wb == rb * T && we == (rb + 1) * T,
+                               rb == rb_first ? 0 : 1, crank, tid);
     }
-    named_bar_sync(2, kConsumerWarps * 32);  // comb is rewritten at the next row block
-    row_block_end<M, ES, CL>(p, smem, s_flag, sum, rb, wb == rb * T && we == (rb + 1) * T,
-                             rb == rb_first ? 0 : 1, crank, tid);
   }
 }
 
@@ -685,15 +845,17 @@ sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, in
 // Thread-block cluster split: each row block is split over S CTAs of one cluster
 // (S <= 16, S <= T, all CTAs within kCtasPerSm per SM), which replaces the global
 // split-K fix-up by a distributed-shared-memory reduction.  Taken when the clusters fill
-// at least 90% of the CTA slots, or when the matrix is small (few row blocks: there the
-// fixed latency of the global fix-up dominates); otherwise stream-K balances better.
+// at least 80% of the CTA slots (measured: on the 172 row blocks of gate/up, 3-CTA
+// clusters filling 85% beat stream-K over all slots), or when the matrix is small (few
+// row blocks: there the fixed latency of the global fix-up dominates); otherwise stream-K
+// balances better.
 int cluster_cc(const sp_matrix* h) {
   const int64_t cap = (int64_t)kCtasPerSm * h->num_sms;
   const int64_t rb = std::max<int32_t>(h->RB, 1);
   int64_t S = std::min<int64_t>(16, cap / rb);
   S = std::min<int64_t>(S, h->T);
   if (S < 2) return 1;
-  const bool fills = 10 * rb * S >= 9 * cap;
+  const bool fills = 10 * rb * S >= 8 * cap;
   const bool small = 8 * rb <= cap;
   return (fills || small) ? (int)S : 1;
 }
@@ -721,7 +883,7 @@ bool cc_plan(const sp_matrix* h, int Mt, int S, CcPlan* pl) {
   // tags (<= 64 B), the warps' partials (warp-per-chunk kernel) and the CTA's FP32
   // partial (cluster mode)
   const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
-  const size_t comb_bytes = (size_t)kConsumerWarps * kRows * Mt * sizeof(float);
+  const size_t comb_bytes = 2 * (size_t)kConsumerWarps * kRows * Mt * sizeof(float) + sizeof(FlushCtl);
   pl->kind = 0;
   size_t ring = kSmemBudget - 256 - 16 - 64 - part_bytes;
   if (Mt <= 4 && (ring - comb_bytes) / pl->slot_bytes >= (size_t)kConsumerWarps) {
