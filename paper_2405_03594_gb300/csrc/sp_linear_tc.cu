@@ -12,9 +12,11 @@
 //
 // CTA (one per SM, persistent, stream-K over work items (token tile, row block, K-tile)):
 //   warp 0 lane 0   producer: cp.async.bulk of each chunk and a TMA tile of x into a
-//                   ring of shared-memory slots (full/empty mbarriers);
+//                   ring of S shared-memory slots; item n uses slot n % S and TMEM A
+//                   stage n % S, and one MMA commit frees both (stage_free[n % S]);
 //   warp 1          TMEM allocation; lane 0 issues the MMAs (4 x K=16 per chunk) and
-//                   commits them to mbarriers that free A stages, ring slots and D;
+//                   commits them to mbarriers that free the stage and, at a segment's
+//                   end, hand D to the epilogue;
 //   warps 2-9       two expander warpgroups taking alternate chunks: thread r of a
 //                   warpgroup owns TMEM lane / chunk row r; it finds its first value by a
 //                   popc prefix sum, expands 64 columns into 32 bf16x2 registers, and
@@ -26,6 +28,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstring>
 #include <mutex>
 
 #include "sp_internal.cuh"
@@ -104,6 +107,23 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
 }
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+// TMA tile store shared -> global (bulk group); rows/columns past the tensor are clipped.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {  // at most N groups still reading shared memory
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy writes of shared memory become visible to the async proxy (TMA)
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row atoms of
@@ -198,7 +218,45 @@ struct TcParams {
   int32_t n_d;        // D buffers in TMEM (1..kMaxDBufs); segment k accumulates in buffer k % n_d
   uint32_t d_cols;    // TMEM columns per D buffer (ntok rounded up to 32)
   uint32_t a_col0;    // first TMEM column of the A stages (n_d * d_cols)
+  int32_t y_tma;      // 1: y is written by TMA stores from a staging tile (needs N % 8 == 0)
+  uint32_t stg_off;   // shared-memory offset of the staging tiles [kExpGroups][2][32][128] bf16
 };
+
+constexpr int kStgTokens = 32;                          // tokens per staged block
+constexpr int kStgBox = 16;                             // tokens per TMA store box
+constexpr uint32_t kStgBytes = kStgTokens * kRows * 2;  // one staging buffer
+
+// Rows rb*128 + r (thread r of the warpgroup) for tokens tok0 .. tok0+nv-1 (nv <= 32, a
+// multiple of 16) of y: bf16(val[i] * sc).  With a y tensor map the warpgroup writes the
+// block into one of its two staging buffers and thread 0 stores it with TMA (16-token
+// boxes; the hardware clips rows past M and columns past N); strided scalar stores of
+// 2-byte values cost ~1.8 us per 32-token block.  Otherwise each thread stores its row.
+__device__ __forceinline__ void store_y_block(const TcParams& tp, const CUtensorMap* tmap_y, uint16_t* stg, int& step,
+                                              const float (&val)[32], float sc, int nv, int64_t tok0, int64_t rb,
+                                              int r, int tid128, int bar) {
+  const LinearParams& p = tp.p;
+  if (tp.y_tma) {
+    uint16_t* buf = stg + (size_t)(step & 1) * (kStgBytes / 2);
+    if (tid128 == 0) bulk_wait_read<1>();  // the store that last read this buffer is done
+    named_bar_sync(bar, 128);
+#pragma unroll
+    for (int i = 0; i < kStgTokens; ++i) buf[i * kRows + r] = float_to_bf16_bits_rn(val[i] * sc);
+    fence_proxy_async_smem();
+    named_bar_sync(bar, 128);
+    if (tid128 == 0) {
+      for (int b0 = 0; b0 < nv; b0 += kStgBox) tma_store_2d(tmap_y, buf + b0 * kRows, (int)(rb * kRows), (int)(tok0 + b0));
+      bulk_commit();
+    }
+    ++step;
+  } else {
+    const int64_t nrow = rb * kRows + r;
+#pragma unroll
+    for (int i = 0; i < kStgTokens; ++i) {
+      const int64_t tok = tok0 + i;
+      if (i < nv && tok < p.M && nrow < p.N) p.y[tok * p.N + nrow] = float_to_bf16_bits_rn(val[i] * sc);
+    }
+  }
+}
 
 // TMEM split for a token tile of ntok columns: D buffers first, A stages after.  Small
 // tiles (decode) leave room for two D buffers and up to 14 A stages, so neither the
@@ -216,15 +274,23 @@ __host__ __device__ inline void tmem_split(int ntok, int* n_a, int* n_d, uint32_
 
 template <int ES>
 __global__ void __launch_bounds__(kThreads, 1)
-    linear_tc_kernel(const __grid_constant__ TcParams tp, const __grid_constant__ CUtensorMap tmap_x) {
+    linear_tc_kernel(const __grid_constant__ TcParams tp, const __grid_constant__ CUtensorMap tmap_x,
+                     const __grid_constant__ CUtensorMap tmap_y) {
   extern __shared__ uint8_t smem_raw[];
   const LinearParams& p = tp.p;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int slots = p.slots;
+  // Ring: item n uses slot n % S and A stage n % S (S = slots <= A stages, even).
+  //   full[s]       chunk and x tile landed (producer's expect_tx + the copies)
+  //   a_full[s]     the four warps of the item's expander warpgroup stored the A stage
+  //   stage_free[s] the item's MMAs completed (one commit): slot and A stage are free.
+  // The expanders read the chunk before arriving on a_full, and the MMAs are issued only
+  // after a_full, so that one commit also covers the expanders' reads of the slot.  An
+  // expander waits only on full[s]: the producer refills a slot only after stage_free,
+  // and with S even a slot's previous item belongs to the same warpgroup.
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)slots * p.slot_bytes);
-  uint64_t* empty = full + slots;
-  uint64_t* a_full = empty + slots;
-  uint64_t* a_empty = a_full + kMaxAStages;
+  uint64_t* stage_free = full + slots;
+  uint64_t* a_full = stage_free + slots;
   // D handshakes.  Segment k (the k-th (token tile, row block) this CTA touches)
   // accumulates in buffer k % n_d, and its epilogue is run by the warpgroup that expanded
   // its last K-tile.  d_full has one barrier per (buffer, warpgroup): a group waits on
@@ -233,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // has finished the previous segment on that buffer).  d_empty has one barrier per
   // buffer: the MMA issuer starts segment k only after the epilogue of segment k - n_d
   // has read that buffer, so those epilogues complete in order.
-  uint64_t* d_full = a_empty + kMaxAStages;               // [kMaxDBufs][kExpGroups]
+  uint64_t* d_full = a_full + slots;                      // [kMaxDBufs][kExpGroups]
   uint64_t* d_empty = d_full + kMaxDBufs * kExpGroups;    // [kMaxDBufs]
   uint32_t* tmem_base_slot = reinterpret_cast<uint32_t*>(d_empty + kMaxDBufs);
   volatile int* s_flag = reinterpret_cast<volatile int*>(tmem_base_slot + 1);  // one per warpgroup
@@ -247,11 +313,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < slots; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 4 + 1);  // four expander warps + one MMA commit
-    }
-    for (int a = 0; a < kMaxAStages; ++a) {
-      mbar_init(&a_full[a], 4);
-      mbar_init(&a_empty[a], 1);
+      mbar_init(&stage_free[s], 1);  // one MMA commit
+      mbar_init(&a_full[s], 4);      // the four warps of an expander warpgroup
     }
     for (int b = 0; b < kMaxDBufs * kExpGroups; ++b) mbar_init(&d_full[b], 1);
     for (int b = 0; b < kMaxDBufs; ++b) mbar_init(&d_empty[b], 4);  // the epilogue warpgroup's four warps
@@ -261,7 +324,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(tmem_base_slot, kTmemCols);
     tmem_relinquish();
   }
-  if (warp == 0 && lane == 0) prefetch_tmap(&tmap_x);
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tmap_x);
+    if (tp.y_tma) prefetch_tmap(&tmap_y);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -299,7 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint64_t o0, o1;
         ow.at(c, &o0, &o1);
         if (lane == 0) {
-          if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+          if (!mbar_wait(&stage_free[s], ph ^ 1u, p.timeout_ns)) {
             set_status(p.status, kStatusTimeout);
             failed = true;
           } else {
@@ -328,9 +394,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       pdl_wait();
       pdl_launch_dependents();
       const uint32_t idesc = idesc_bf16(tp.ntok);
-      const int n_a = tp.n_a, n_d = tp.n_d;
-      int s = 0, as = 0;
-      uint32_t ph = 0, aph = 0;
+      const int n_d = tp.n_d;
+      int s = 0;
+      uint32_t ph = 0;
       int k = -1;  // local segment number
       int db = 0;  // D buffer of segment k
       uint32_t d_taddr = tmem;
@@ -357,30 +423,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           dead = true;
           set_status(p.status, kStatusTimeout);
         }
-        if (!dead && !mbar_wait(&a_full[as], aph, p.timeout_ns)) {
+        if (!dead && !mbar_wait(&a_full[s], ph, p.timeout_ns)) {
           dead = true;
           set_status(p.status, kStatusTimeout);
         }
         if (!dead) {
           tc_fence_after();
           const uint32_t b_saddr = smem_u32(smem + (size_t)s * p.slot_bytes);
-          const uint32_t a_taddr = tmem + tp.a_col0 + (uint32_t)as * 32u;
+          const uint32_t a_taddr = tmem + tp.a_col0 + (uint32_t)s * 32u;
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk) {
             const uint64_t bdesc = smem_desc_sw128(b_saddr + (uint32_t)kk * 32u);
             mma_ts(d_taddr, a_taddr + (uint32_t)kk * 8u, bdesc, idesc, (seg_first && kk == 0) ? 0u : 1u);
           }
-          mma_commit(&empty[s]);
-          mma_commit(&a_empty[as]);
+          mma_commit(&stage_free[s]);
           if (seg_last) mma_commit(&d_full[db * kExpGroups + (int)((w - w0) % kExpGroups)]);
         }
         if (++s == slots) {
           s = 0;
           ph ^= 1u;
-        }
-        if (++as == n_a) {
-          as = 0;
-          aph ^= 1u;
         }
       }
     }
@@ -394,19 +455,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = (uint32_t)(q * 32) << 16;
     const int tid128 = (warp - kExpWarp0 - 4 * grp) * 32 + lane;
     bool dead = false;
-    const int n_a = tp.n_a;
     const int64_t sg_first = w0 / T;
-    // ring positions of item n = grp, grp + kExpGroups, ... (slots, n_a >= kExpGroups)
-    int s = grp, as = grp;
-    uint32_t ph = 0, aph = 0;
+    // ring position of item n = grp, grp + kExpGroups, ... (slots >= kExpGroups)
+    int s = grp;
+    uint32_t ph = 0;
     int t = (int)((w0 + grp) % T);  // K-tile of item w
     uint32_t dph_bits = 0;          // phase parity of this group's d_full barrier, per buffer
+    uint16_t* stg = reinterpret_cast<uint16_t*>(smem + tp.stg_off) + (size_t)grp * kStgBytes;  // 2 buffers
+    int stg_step = 0;
+    const int bar = 1 + grp;        // named barrier of this warpgroup
     for (int64_t w = w0 + grp, n = grp; w < w1; w += kExpGroups, n += kExpGroups) {
       const bool seg_last = (w + 1 == w1) || t == T - 1;
       for (t += kExpGroups; t >= T;) t -= T;
       if (!dead) {
-        bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
-        if (ok && n >= n_a) ok = __all_sync(0xffffffffu, mbar_wait(&a_empty[as], aph ^ 1u, p.timeout_ns));
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
         if (!ok) {
           dead = true;
           set_status(p.status, kStatusTimeout);
@@ -438,22 +500,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t pa = vbase + (uint32_t)(e0 * ES);   // stream of columns 0-31
         uint32_t pb = pa + (uint32_t)(plo * ES);     // stream of columns 32-63
         expand_pair<ES, 0>(mlo, mhi, pa, pb, o);
-        tmem_store32(tmem + lane_base + tp.a_col0 + (uint32_t)as * 32u, o);
+        tmem_store32(tmem + lane_base + tp.a_col0 + (uint32_t)s * 32u, o);
         tmem_store_wait();
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&a_full[as]);
-        mbar_arrive(&empty[s]);
-      }
+      if (lane == 0) mbar_arrive(&a_full[s]);
       if ((s += kExpGroups) >= slots) {
         s -= slots;
         ph ^= 1u;
-      }
-      if ((as += kExpGroups) >= n_a) {
-        as -= n_a;
-        aph ^= 1u;
       }
 
       // ---------------------------------------------------------- segment end: epilogue
@@ -489,23 +544,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_load32(d_taddr + lane_base + (uint32_t)c0, v);
           tmem_load_wait();
         }
+        const int nv = tp.ntok - c0 < 32 ? tp.ntok - c0 : 32;  // ntok is a multiple of 16
+        if (complete) {
+          float a[32];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          if (c0 + i >= tp.ntok) break;  // ntok is a multiple of 16, not always of 32
-          const int64_t tok = mtile * tp.ntok + c0 + i;
-          const float a = __uint_as_float(v[i]);
-          if (complete) {
-            if (tok < p.M && nrow < p.N) p.y[tok * p.N + nrow] = float_to_bf16_bits_rn(a * sc);
-          } else {
-            __stcg(wsp + (int64_t)(c0 + i) * kRows + r, a);
-          }
+          for (int i = 0; i < 32; ++i) a[i] = __uint_as_float(v[i]);
+          store_y_block(tp, &tmap_y, stg, stg_step, a, sc, nv, mtile * tp.ntok + c0, rb, r, tid128, bar);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nv) __stcg(wsp + (int64_t)(c0 + i) * kRows + r, __uint_as_float(v[i]));
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&d_empty[db]);
       if (!complete) {
-        const int bar = 1 + grp;
         __threadfence();
         named_bar_sync(bar, 128);
         const int64_t i_first = owner_of(seg_begin, p.W, p.G);
@@ -531,12 +585,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               for (int i = 0; i < 32; ++i)
                 if (c0 + i < tp.ntok) sum[i] += __ldcg(src + (int64_t)i * kRows);
             }
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int64_t tok = mtile * tp.ntok + c0 + i;
-              if (c0 + i < tp.ntok && tok < p.M && nrow < p.N)
-                p.y[tok * p.N + nrow] = float_to_bf16_bits_rn(sum[i] * sc);
-            }
+            const int nv = tp.ntok - c0 < 32 ? tp.ntok - c0 : 32;
+            store_y_block(tp, &tmap_y, stg, stg_step, sum, sc, nv, mtile * tp.ntok + c0, rb, r, tid128, bar);
           }
           if (tid128 == 0) atomicExch(ctr, 0);
         }
@@ -544,6 +594,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
+  if (tp.y_tma && warp >= kExpWarp0 && ((warp - kExpWarp0) & 3) == 0 && lane == 0) bulk_wait_all();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -581,7 +632,8 @@ int ntok_for(int64_t M) {
 }
 
 template <int ES>
-sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, size_t smem, cudaStream_t stream) {
+sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtensorMap& map_y, size_t smem,
+                       cudaStream_t stream) {
   auto kern = linear_tc_kernel<ES>;
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -604,7 +656,7 @@ sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, size_t smem, 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, kern, tp, map) != cudaSuccess) {
+  if (cudaLaunchKernelEx(&cfg, kern, tp, map, map_y) != cudaSuccess) {
     cudaGetLastError();
     return SP_ERR_CUDA;
   }
@@ -654,15 +706,21 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   tp.chunk_off = (tp.b_bytes + 1023u) / 1024u * 1024u;
   p.chunk_region = (uint32_t)((h->max_chunk + 1023) / 1024 * 1024);
   p.slot_bytes = tp.chunk_off + p.chunk_region;
-  // base alignment + barriers (2 per slot, 2 per A stage, 2 for D), TMEM address, flag
-  const size_t tail =
-      1024 + 8 * (2 * kMaxSlots + 2 * kMaxAStages + kMaxDBufs * (kExpGroups + 1)) + 4 + 4 * kExpGroups + 16;
-  // an even number of slots: the expander warpgroups take alternate items, so a slot's
-  // previous item then belongs to the warpgroup now waiting on it, which keeps the parity
-  // wait on the slot's full barrier exact
-  const int slots = (int)std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes) & ~1;
+  // base alignment + barriers (3 per slot, D handshakes), TMEM address, flags, and (TMA
+  // stores of y) the staging tiles, 1024-byte aligned
+  tp.y_tma = (h->N % 8 == 0) ? 1 : 0;
+  const size_t ctl_bytes = 8 * (3 * kMaxSlots + kMaxDBufs * (kExpGroups + 1)) + 4 + 4 * kExpGroups + 16;
+  const size_t stg_bytes = tp.y_tma ? (size_t)kExpGroups * 2 * kStgBytes : 0;
+  const size_t tail = 1024 + (ctl_bytes + 1023) / 1024 * 1024 + stg_bytes;
+  // S = slots = A stages in use, an even number: the expander warpgroups take alternate
+  // items, so a slot's previous item belongs to the warpgroup now waiting on it, which
+  // keeps the parity wait on the slot's full barrier exact
+  const int slots = (int)std::min<size_t>(std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes),
+                                          (size_t)tp.n_a) &
+                    ~1;
   if (slots < 2) return SP_ERR_UNSUPPORTED;
   p.slots = slots;
+  tp.stg_off = (uint32_t)((size_t)slots * p.slot_bytes + (ctl_bytes + 1023) / 1024 * 1024);
   // at least 116 KB so that two CTAs never share an SM (each allocates 512 TMEM columns)
   const size_t smem = std::max<size_t>((size_t)slots * p.slot_bytes + tail, 116 * 1024);
 
@@ -677,7 +735,21 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return SP_ERR_CUDA;
-  return h->esize == 2 ? launch_tc_es<2>(tp, map, smem, stream) : launch_tc_es<1>(tp, map, smem, stream);
+  // y [M, N] bf16 written by TMA stores in boxes of 128 rows x 16 tokens (needs a row pitch
+  // that is a multiple of 16 bytes); otherwise the epilogue stores scalars
+  CUtensorMap map_y;
+  memset(&map_y, 0, sizeof(map_y));
+  if (tp.y_tma) {
+    const cuuint64_t ydim[2] = {(cuuint64_t)h->N, (cuuint64_t)M};
+    const cuuint64_t ystride[1] = {(cuuint64_t)h->N * 2};
+    const cuuint32_t ybox[2] = {(cuuint32_t)kRows, (cuuint32_t)kStgBox};
+    if (encode(&map_y, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, y, ydim, ystride, ybox, estride,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return SP_ERR_CUDA;
+  }
+  return h->esize == 2 ? launch_tc_es<2>(tp, map, map_y, smem, stream)
+                       : launch_tc_es<1>(tp, map, map_y, smem, stream);
 }
 
 }  // namespace sp
