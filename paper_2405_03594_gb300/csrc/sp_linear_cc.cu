@@ -255,8 +255,44 @@ __device__ __forceinline__ void row_dot(uint32_t lo, uint32_t hi, int plo, int p
     }
 #pragma unroll
     for (int m = 0; m < M; ++m) acc[m] += accl[m] + acch[m];
+  } else if constexpr (ES == 1 && M <= 4) {
+    // int8 values, small batch: each chain keeps its own accumulators; a value is one
+    // signed byte load and one int -> float conversion, x[m, j] is widened from bf16 by a
+    // shift, and the product (int8 x bf16, exact in FP32) is added with an FP32 FMA
+    float accl[M], acch[M];
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      accl[m] = 0.f;
+      acch[m] = 0.f;
+    }
+    const int8_t* v8 = reinterpret_cast<const int8_t*>(vals);
+#pragma unroll 2
+    for (int q = 0; q < iters; ++q) {
+      const int jl = msb32(lo), jh = msb32(hi);
+      lo = clear_bit(lo, jl);
+      hi = clear_bit(hi, jh);
+      // unconditional loads (an exhausted chain reads at most 32 bytes below the row's first
+      // value, still inside the chunk's mask area); only the FMAs are predicated
+      const float wl = (float)v8[top_lo - q];
+      const float wh = (float)v8[top_hi - q];
+#pragma unroll
+      for (int r = 0; r < MP; ++r) {
+        const uint32_t xl = __shfl_sync(0xffffffffu, XL[r], jl);
+        const uint32_t xh = __shfl_sync(0xffffffffu, XH[r], jh);
+        if (jl >= 0) {
+          accl[2 * r] = fmaf(wl, __uint_as_float(xl << 16), accl[2 * r]);
+          if (2 * r + 1 < M) accl[2 * r + 1] = fmaf(wl, __uint_as_float(xl & 0xffff0000u), accl[2 * r + 1]);
+        }
+        if (jh >= 0) {
+          acch[2 * r] = fmaf(wh, __uint_as_float(xh << 16), acch[2 * r]);
+          if (2 * r + 1 < M) acch[2 * r + 1] = fmaf(wh, __uint_as_float(xh & 0xffff0000u), acch[2 * r + 1]);
+        }
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < M; ++m) acc[m] += accl[m] + acch[m];
   } else {
-    // larger batches (or int8 values): one value per chain step, one accumulator set
+    // larger batches: one value per chain step, one accumulator set
 #pragma unroll 2
     for (int q = 0; q < iters; ++q) {
       const int jl = msb32(lo), jh = msb32(hi);
