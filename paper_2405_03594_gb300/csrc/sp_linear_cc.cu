@@ -351,13 +351,24 @@ __device__ __forceinline__ void row_block_end(const LinearParams& p, uint8_t* sm
 #pragma unroll
       for (int m = 0; m < M; ++m) sum[m] = acc[m];
       const uint32_t base = smem_u32(part) + 4u * (uint32_t)tid;
-      for (int r = 1; r < p.cluster; ++r) {
-        const uint32_t rb_addr = cluster_map(base, (uint32_t)r);
-        float v[M];
+      // the other ranks' partials, kR ranks' loads in flight at a time; the adds stay in
+      // rank order
+      constexpr int kR = M <= 2 ? 4 : 2;
+      for (int r0 = 1; r0 < p.cluster; r0 += kR) {
+        float v[kR][M];
 #pragma unroll
-        for (int m = 0; m < M; ++m) v[m] = ld_cluster_f32(rb_addr + 4u * (uint32_t)(m * kRows));
+        for (int u = 0; u < kR; ++u)
+          if (r0 + u < p.cluster) {
+            const uint32_t rb_addr = cluster_map(base, (uint32_t)(r0 + u));
 #pragma unroll
-        for (int m = 0; m < M; ++m) sum[m] += v[m];
+            for (int m = 0; m < M; ++m) v[u][m] = ld_cluster_f32(rb_addr + 4u * (uint32_t)(m * kRows));
+          }
+#pragma unroll
+        for (int u = 0; u < kR; ++u)
+          if (r0 + u < p.cluster) {
+#pragma unroll
+            for (int m = 0; m < M; ++m) sum[m] += v[u][m];
+          }
       }
       if (n < p.N) {
 #pragma unroll
