@@ -37,6 +37,50 @@ sp_status sp_residual_add(void* h, const void* a, const void* r, int64_t M, int6
 /* out[m, j] = bf16(g[m, j] * g[m, F + j]) for j < F; g [M, 2F], out [M, F]; F % 8 == 0. */
 sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* stream);
 
+
+/* ---------------------------------------------------------------- chained decode step
+ * A chain of sparse linears run by one persistent launch (a decode step through the
+ * layers of a model).  Linear k computes acc = x_k . (W_k o Mask_k)^T (FP32 accumulation;
+ * Sec. 2.4.2's compressed submatrices streamed from global memory and expanded on chip)
+ * and writes it through one of the epilogues below.  Every linear waits for the previous
+ * one to be complete (its x may be any earlier output), while the compressed weights of
+ * all linears stream from HBM without a break between linears.  Results equal those of
+ * the corresponding sp_linear calls and sp_stack glue up to FP32 summation order, and are
+ * bitwise repeatable for a given (chain, m, device). */
+typedef enum sp_chain_epilogue {
+  SP_EPI_STORE = 0,        /* y[m, n] = bf16(acc)                                          */
+  SP_EPI_RESIDUAL = 1,     /* y[m, n] = bf16((y[m, n] + bf16(acc)) + r[n]), in place      */
+  SP_EPI_PAIR_PRODUCT = 2  /* rows 2j and 2j+1 (N even): y[m, j] = bf16(bf16(acc_2j) *
+                              bf16(acc_2j+1)) -- the gate*up product when the rows of the
+                              fused gate/up weight are interleaved (gate_j, up_j)          */
+} sp_chain_epilogue;
+
+typedef struct sp_chain_op {
+  const sp_matrix* w;  /* compressed weight [N, K] (INT8: bf16(acc) is bf16(s[n] * acc))   */
+  const void* x;       /* bf16 input [m, K] with row stride ldx elements (ldx >= K)        */
+  int64_t ldx;
+  void* y;             /* bf16 output, row stride ldy (>= N, or >= N/2 for the pair product) */
+  int64_t ldy;
+  const void* r;       /* bf16 [N] residual vector for SP_EPI_RESIDUAL, else NULL           */
+  int32_t epilogue;    /* sp_chain_epilogue */
+  int32_t reserved;    /* 0 */
+} sp_chain_op;
+
+/* Workspace bytes that sp_chain_run needs on the current device (0 for m == 0). */
+sp_status sp_chain_workspace_size(int64_t m, size_t* bytes);
+
+/* Run ops[0], ops[1], ..., ops[n_ops - 1] in order for m batch rows (1 <= m <= 4;
+ * SP_ERR_UNSUPPORTED above).  All weights live on the current device and hold the same
+ * value type (bf16 or INT8).  x, y and r are 2-byte aligned (any row stride); the workspace
+ * is 16-byte aligned.  The workspace (sp_chain_workspace_size bytes) is zero-filled before
+ * its first use, and every call leaves it ready for the next; calls that share it must be
+ * ordered on one stream.  After SP_ERR_TIMEOUT from sp_check, zero it again.  Each group
+ * of up to 160 linears is one launch (all its CTAs resident at once, launched
+ * cooperatively); the launch allocates nothing and does not synchronise the host.
+ * m == 0 or n_ops == 0 returns SP_OK without a launch. */
+sp_status sp_chain_run(const sp_chain_op* ops, int32_t n_ops, int64_t m, void* workspace_dev, size_t workspace_bytes,
+                       void* stream);
+
 #ifdef __cplusplus
 }
 #endif

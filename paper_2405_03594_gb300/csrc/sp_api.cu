@@ -171,17 +171,21 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
   c->ctx = alloc_ctx;
   c->d_buf = nullptr;
   c->d_off = nullptr;
+  c->d_qidx = nullptr;
   c->d_scale = nullptr;
   const size_t off_bytes = ((size_t)h->RB * h->T + 1) * sizeof(uint64_t);
   cudaStream_t s = (cudaStream_t)stream;
   sp_status st = SP_OK;
   c->d_buf = (uint8_t*)dev_alloc(c, (size_t)std::max<uint64_t>(h->bytes, 16));
   c->d_off = (uint64_t*)dev_alloc(c, off_bytes);
+  c->d_qidx = (uint64_t*)dev_alloc(c, off_bytes - sizeof(uint64_t));
   if (h->d_scale) c->d_scale = (float*)dev_alloc(c, (size_t)h->N * sizeof(float));
-  if (!c->d_buf || !c->d_off || (h->d_scale && !c->d_scale)) {
+  if (!c->d_buf || !c->d_off || !c->d_qidx || (h->d_scale && !c->d_scale)) {
     st = SP_ERR_OUT_OF_MEMORY;
   } else if (cudaMemcpyAsync(c->d_buf, h->d_buf, h->bytes, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
              cudaMemcpyAsync(c->d_off, h->d_off, off_bytes, cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+             cudaMemcpyAsync(c->d_qidx, h->d_qidx, off_bytes - sizeof(uint64_t), cudaMemcpyDeviceToDevice, s) !=
+                 cudaSuccess ||
              (h->d_scale && cudaMemcpyAsync(c->d_scale, h->d_scale, (size_t)h->N * sizeof(float),
                                             cudaMemcpyDeviceToDevice, s) != cudaSuccess) ||
              cudaStreamSynchronize(s) != cudaSuccess) {
@@ -191,6 +195,7 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
     cudaGetLastError();
     dev_free(c, c->d_buf);
     dev_free(c, c->d_off);
+    dev_free(c, c->d_qidx);
     dev_free(c, c->d_scale);
     delete c;
     return st;
@@ -206,6 +211,7 @@ sp_status sp_free(sp_matrix* h) {
   h->magic = 0;
   dev_free(h, h->d_buf);
   dev_free(h, h->d_off);
+  dev_free(h, h->d_qidx);
   dev_free(h, h->d_scale);
   delete h;
   return SP_OK;

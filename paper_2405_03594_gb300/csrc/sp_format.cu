@@ -41,9 +41,13 @@ __device__ __forceinline__ int block_excl_scan_128(int v, int* total, int* s_war
   return base + incl - v;
 }
 
+// Also writes the chunk's quarter index (kept entries before rows 32, 64 and 96, and in the
+// whole chunk; 16 bits each) and raises *max_quarter to its largest quarter count.
 __global__ void __launch_bounds__(kRows) count_kernel(const uint8_t* __restrict__ mask, int64_t N, int64_t K, int T,
-                                                      uint64_t* __restrict__ masks_out, int* __restrict__ cnt) {
+                                                      uint64_t* __restrict__ masks_out, int* __restrict__ cnt,
+                                                      uint64_t* __restrict__ qidx, int* __restrict__ max_quarter) {
   __shared__ int s_warp[kRows / 32];
+  __shared__ int s_q[kRows / 32];
   const int64_t c = blockIdx.x;
   const int64_t rb = c / T, t = c % T;
   const int r = threadIdx.x;
@@ -61,8 +65,15 @@ __global__ void __launch_bounds__(kRows) count_kernel(const uint8_t* __restrict_
   }
   masks_out[c * kRows + r] = m;
   int total;
-  block_excl_scan_128(__popcll(m), &total, s_warp);
-  if (r == 0) cnt[c] = total;
+  const int excl = block_excl_scan_128(__popcll(m), &total, s_warp);
+  if ((r & 31) == 0) s_q[r >> 5] = excl;
+  __syncthreads();
+  if (r == 0) {
+    cnt[c] = total;
+    qidx[c] = (uint64_t)s_q[1] | ((uint64_t)s_q[2] << 16) | ((uint64_t)s_q[3] << 32) | ((uint64_t)total << 48);
+    const int q = max(max(s_q[1] - s_q[0], s_q[2] - s_q[1]), max(s_q[3] - s_q[2], total - s_q[3]));
+    atomicMax(max_quarter, q);
+  }
 }
 
 // meta[0] = total bytes, meta[1] = largest chunk, meta[2] = kept entries
@@ -228,12 +239,19 @@ sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t
   int* d_cnt = (int*)dev_alloc(h, (size_t)C * sizeof(int));
   uint64_t* d_meta = (uint64_t*)dev_alloc(h, 4 * sizeof(uint64_t));
   h->d_off = (uint64_t*)dev_alloc(h, (size_t)(C + 1) * sizeof(uint64_t));
+  h->d_qidx = (uint64_t*)dev_alloc(h, (size_t)C * sizeof(uint64_t));
   uint64_t meta[4] = {0, 0, 0, 0};
-  if (!d_masks || !d_cnt || !d_meta || !h->d_off) {
+  if (!d_masks || !d_cnt || !d_meta || !h->d_off || !h->d_qidx) {
     st = SP_ERR_OUT_OF_MEMORY;
     goto fail;
   }
-  count_kernel<<<(unsigned)C, kRows, 0, stream>>>(mask, N, K, h->T, d_masks, d_cnt);
+  // meta[3] holds the largest quarter count (count_kernel's atomicMax target)
+  if (cudaMemsetAsync(d_meta, 0, 4 * sizeof(uint64_t), stream) != cudaSuccess) {
+    st = SP_ERR_CUDA;
+    goto fail;
+  }
+  count_kernel<<<(unsigned)C, kRows, 0, stream>>>(mask, N, K, h->T, d_masks, d_cnt, h->d_qidx,
+                                                   reinterpret_cast<int*>(d_meta + 3));
   scan_kernel<<<1, 1024, 0, stream>>>(d_cnt, C, h->esize, h->d_off, d_meta);
   if (cudaGetLastError() != cudaSuccess) {
     st = SP_ERR_CUDA;
@@ -247,6 +265,7 @@ sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t
   h->bytes = meta[0];
   h->max_chunk = meta[1];
   h->nnz = (int64_t)meta[2];
+  h->max_quarter = (uint32_t)(meta[3] & 0xffffffffu);
   h->d_buf = (uint8_t*)dev_alloc(h, (size_t)std::max<uint64_t>(h->bytes, 16));
   if (!h->d_buf) {
     st = SP_ERR_OUT_OF_MEMORY;
@@ -284,6 +303,7 @@ fail:
   dev_free(h, d_cnt);
   dev_free(h, d_meta);
   dev_free(h, h->d_off);
+  dev_free(h, h->d_qidx);
   dev_free(h, h->d_buf);
   dev_free(h, h->d_scale);
   delete h;

@@ -20,8 +20,11 @@ struct sp_matrix {
   int64_t nnz;
   uint64_t bytes;
   uint64_t max_chunk;
+  uint32_t max_quarter;  // most kept entries in one 32-row quarter of a chunk
   uint8_t* d_buf;
   uint64_t* d_off;
+  uint64_t* d_qidx;      // per chunk: kept entries before rows 32, 64, 96 and in all 128 rows
+                         // (16 bits each, low to high), derived from the masks at compression
   float* d_scale;
   sp_alloc_fn alloc;
   sp_free_fn free_fn;
@@ -123,6 +126,28 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   while (true) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > timeout_ns) return false;
+  }
+}
+// try_wait with a suspend-time hint: the thread sleeps until the phase completes or about
+// `hint_ns` pass, instead of returning at once (fewer issue slots spent waiting).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait as mbar_wait, sleeping in the hardware between checks.
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (true) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if (global_ns() - t0 > timeout_ns) return false;
   }
 }

@@ -27,7 +27,7 @@ STATUS = {
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
            "sp_linear_noalloc",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
-           "sp_copy_columns", "sp_residual_add", "sp_mul_halves"]
+           "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_chain_workspace_size", "sp_chain_run"]
 
 
 KERNELS = {0: "", 1: "linear_cc_kernel", 2: "linear_ccw_kernel", 3: "linear_tc_kernel"}  # SP_KERNEL_*
@@ -44,6 +44,15 @@ class SpInfo(ctypes.Structure):
                 ("row_blocks", ctypes.c_int64), ("dtype", ctypes.c_int32), ("device", ctypes.c_int32),
                 ("nnz", ctypes.c_int64), ("bytes", ctypes.c_uint64), ("max_chunk_bytes", ctypes.c_uint64),
                 ("scale_bytes", ctypes.c_uint64)]
+
+
+EPILOGUES = {"store": 0, "residual": 1, "pair_product": 2}  # sp_chain_epilogue
+
+
+class SpChainOp(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("x", ctypes.c_void_p), ("ldx", ctypes.c_int64), ("y", ctypes.c_void_p),
+                ("ldy", ctypes.c_int64), ("r", ctypes.c_void_p), ("epilogue", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p)
@@ -69,6 +78,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_copy_columns.argtypes = [P, P, I64, I64, I64, I64, P]
     lib.sp_residual_add.argtypes = [P, P, P, I64, I64, P]
     lib.sp_mul_halves.argtypes = [P, P, I64, I64, P]
+    lib.sp_chain_workspace_size.argtypes = [I64, ctypes.POINTER(SZ)]
+    lib.sp_chain_run.argtypes = [ctypes.POINTER(SpChainOp), ctypes.c_int32, I64, P, SZ, P]
     lib.sp_status_string.argtypes = [ctypes.c_int]
     lib.sp_status_string.restype = ctypes.c_char_p
     for name in EXPORTS:
@@ -255,6 +266,35 @@ def mul_halves(out: torch.Tensor, g: torch.Tensor, stream=None) -> torch.Tensor:
     M, F = out.shape
     _check(_lib.sp_mul_halves(_ptr(out), _ptr(g), M, F, _stream(stream)), "sp_mul_halves")
     return out
+
+
+class Chain:
+    """A fixed chain of sparse linears (sp_chain_run): op k reads its x only once op k-1 is
+    complete.  Each op is (matrix, x view, y view, epilogue, r); x and y are 2-D bf16 views
+    with unit column stride (row stride = their stride(0)).  The ctypes op array is built
+    once; run() is one library call per group of up to 160 linears."""
+
+    def __init__(self, ops, m: int):
+        self.m = m
+        self._keep = []
+        arr = (SpChainOp * max(len(ops), 1))()
+        for i, (mat, x, y, epi, r) in enumerate(ops):
+            assert x.dtype == torch.bfloat16 and y.dtype == torch.bfloat16 and x.stride(1) == 1 and y.stride(1) == 1
+            assert x.shape[0] >= m and y.shape[0] >= m and x.shape[1] == mat.k
+            assert y.shape[1] == (mat.n // 2 if epi == "pair_product" else mat.n)
+            arr[i] = SpChainOp(mat.handle, x.data_ptr(), x.stride(0), y.data_ptr(), y.stride(0),
+                               0 if r is None else r.data_ptr(), EPILOGUES[epi], 0)
+            self._keep.append((mat, x, y, r))
+        self._ops = arr
+        self.n_ops = len(ops)
+        b = ctypes.c_size_t()
+        _check(_lib.sp_chain_workspace_size(m, ctypes.byref(b)), "sp_chain_workspace_size")
+        dev = torch.device("cuda", torch.cuda.current_device())
+        self.workspace = torch.zeros(max(int(b.value), 256), dtype=torch.uint8, device=dev)
+
+    def run(self, stream=None):
+        _check(_lib.sp_chain_run(self._ops, self.n_ops, self.m, _ptr(self.workspace), self.workspace.numel(),
+                                 _stream(stream)), "sp_chain_run")
 
 
 def check(stream=None):

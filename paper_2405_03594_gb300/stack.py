@@ -12,6 +12,12 @@ Per layer, four fused sparse linears and the elementwise glue of include/sp_stac
 All arithmetic runs in libsp kernels; PyTorch only holds the buffers.  The layers are
 device copies of one seeded layer (each its own HBM buffers), so a step streams the
 full 32-layer weight set.  `capture()` records one step as a single CUDA graph.
+
+`ChainStack` runs the same step (for batches of up to 4 rows) as one persistent launch of
+sp_chain_run: the glue is fused into the linears' epilogues (v is read in place from
+qkv; h + o(v) + r and h + down(a) + r' are residual epilogues), and the gate/up weight is
+stored with its rows interleaved (gate_j, up_j) so that the gate*up product is the pair
+epilogue of one row block.
 """
 from __future__ import annotations
 
@@ -130,3 +136,84 @@ class LinearStack:
             self.step(M, reset=True)
         torch.cuda.synchronize()
         return g
+
+
+def interleave_rows(a: np.ndarray, half: int) -> np.ndarray:
+    """Rows [r_0, ..., r_{F-1}, r_F, ..., r_{2F-1}] -> [r_0, r_F, r_1, r_{F+1}, ...]."""
+    out = np.empty_like(a)
+    out[0::2] = a[:half]
+    out[1::2] = a[half:]
+    return out
+
+
+class ChainStack:
+    """The 32-layer linear stack as one sp_chain_run call per decode step (m <= 4 rows)."""
+
+    def __init__(self, layers: int = 32, pct: int = 70, int8: bool = False, max_m: int = 4, seed: int = 0,
+                 device=None, host=None):
+        self.dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+        self.layers, self.max_m = layers, max_m
+        self.host = host_layer(pct, int8, seed) if host is None else host
+        self.mats = {}
+        for name in SHAPES:
+            vals, mask, s = self.host[name]
+            if name == "gate_up":
+                vals, mask = interleave_rows(vals, D_FF), interleave_rows(mask, D_FF)
+                s = None if s is None else interleave_rows(s, D_FF)
+            if s is not None:
+                h0 = sp.compress(torch.from_numpy(np.ascontiguousarray(vals)).to(self.dev),
+                                 torch.from_numpy(np.ascontiguousarray(mask)).to(self.dev),
+                                 torch.from_numpy(np.ascontiguousarray(s)).to(self.dev))
+            else:
+                h0 = sp.compress(torch.from_numpy(np.ascontiguousarray(vals).view(np.int16)).to(self.dev)
+                                 .view(torch.bfloat16), torch.from_numpy(np.ascontiguousarray(mask)).to(self.dev))
+            self.mats[name] = [h0] + [h0.clone() for _ in range(layers - 1)]
+        g = synth.rng(seed, 0, 9, synth.STREAM_RESID)
+        r = synth.activations(2 * layers, D_MODEL, g)
+        rt = torch.from_numpy(r.view(np.int16)).to(self.dev).view(torch.bfloat16)
+        self.r1 = [rt[2 * l].contiguous() for l in range(layers)]
+        self.r2 = [rt[2 * l + 1].contiguous() for l in range(layers)]
+        bf = dict(dtype=torch.bfloat16, device=self.dev)
+        self.h = torch.zeros((max_m, D_MODEL), **bf)
+        self.x0 = torch.zeros((max_m, D_MODEL), **bf)
+        self.qkv = torch.empty((max_m, 3 * D_MODEL), **bf)
+        self.a = torch.empty((max_m, D_FF), **bf)
+        self._chains = {}
+        torch.cuda.synchronize()
+
+    def weight_bytes(self) -> int:
+        return self.layers * sum(int(self.mats[n][0].info.bytes) + int(self.mats[n][0].info.scale_bytes)
+                                 for n in SHAPES)
+
+    def ops(self, M: int):
+        """The chain of one decode step: four linears per layer."""
+        h, qkv, a = self.h[:M], self.qkv[:M], self.a[:M]
+        v = qkv[:, 2 * D_MODEL:]
+        out = []
+        for l in range(self.layers):
+            out.append((self.mats["qkv"][l], h, qkv, "store", None))
+            out.append((self.mats["o"][l], v, h, "residual", self.r1[l]))
+            out.append((self.mats["gate_up"][l], h, a, "pair_product", None))
+            out.append((self.mats["down"][l], a, h, "residual", self.r2[l]))
+        return out
+
+    def chain(self, M: int) -> "sp.Chain":
+        if M not in self._chains:
+            self._chains[M] = sp.Chain(self.ops(M), M)
+        return self._chains[M]
+
+    def set_input(self, x: torch.Tensor):
+        M = x.shape[0]
+        self.x0[:M].copy_(x)
+        self.h[:M].copy_(x)
+
+    def step(self, M: int, stream=None, reset: bool = True):
+        """One decode step for the first M rows of self.h (in place): two library launches
+        (the copy of the saved input when reset=True, then the whole chain)."""
+        c = self.chain(M)
+        if reset:
+            sp.copy_columns(self.h[:M], self.x0[:M], 0, stream=stream)
+        c.run(stream=stream)
+
+    def launches_per_step(self, M: int, reset: bool = True) -> int:
+        return (4 * self.layers + 159) // 160 + (1 if reset else 0)
