@@ -1,15 +1,15 @@
 #!/usr/bin/env python
 """Decode throughput of the Llama-2-7B sparse linear stack on GB300.
 
-A step is one decode step through the linear layers of all 32 Llama-2-7B layers,
-chained as in the model: per layer the fused qkv (4096->12288), o (4096->4096, added to
-the residual stream h with a fixed vector r), fused gate/up (4096->22016, reduced to
-gate*up) and down (11008->4096, added to h with r'); 70% unstructured per-row magnitude
-sparsity, bf16 weights in the bitmask-compressed format, h bf16 [M, 4096], FP32
-accumulation.  The whole step is one sp_chain_run launch (plus the copy of the step's
-input into h).  tok/s = M / step time.  The 32 layers are 32 distinct device copies of
-one seeded layer, so every step streams 4.7 GB (> L2) of compressed weights from HBM.
-Secondary sections: every linear as its own launch (per shape), the INT8 stack, prefill.
+A step is one decode step through the linear layers of all 32 Llama-2-7B layers:
+per layer the fused qkv (4096->12288), o (4096->4096), fused gate/up (4096->22016)
+and down (11008->4096) projections, 70% unstructured per-row magnitude sparsity,
+bf16 weights in the bitmask-compressed format, x bf16 [M, K], FP32 accumulation,
+bf16 y.  tok/s = M / step time.  The 32 layers are 32 distinct device copies of one
+seeded layer, so every step streams 4.7 GB (> L2) of compressed weights from HBM.
+Further sections: the same step with its elementwise glue (residual adds, gate*up) as one
+persistent sp_chain_run launch and as a CUDA graph of separate launches; the INT8 stack;
+prefill.
 
   python bench.py [--gpus N --steps K --warmup W --m M]        our CUDA path
   python bench.py --impl reference ...                          the float64 CPU oracle
@@ -50,7 +50,7 @@ def parse():
     ap.add_argument("--sweep", default="1,4,16", help="extra batch sizes reported under per_m ('' = none)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle leg")
     ap.add_argument("--no-stack", action="store_true", help="skip the INT8 32-layer stack section")
-    ap.add_argument("--no-per-linear", action="store_true", help="skip the per-linear (one launch per linear) section")
+    ap.add_argument("--no-chain", action="store_true", help="skip the chained-step (glue included) section")
     ap.add_argument("--layers", type=int, default=32, help="profiling aid (--single chain): layers in the chain")
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
@@ -341,11 +341,9 @@ def run_reference(args):
     line = {"metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, Llama-2-7B shapes)", "impl": "reference",
-            "config": {"workload": f"llama2-7b decode step through the linear stack: {LAYERS} layers x (qkv "
-                                   f"4096->12288, o 4096->4096 + residual, gate_up 4096->22016 -> gate*up, down "
-                                   f"11008->4096 + residual), chained, {args.pct}% per-row magnitude sparsity, bf16 "
-                                   f"bitmask format, decode M={args.m}, one persistent launch per step",
-                       "M": args.m, "layers": LAYERS, "sparsity_pct": args.pct},
+            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
+                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
+                                   f"sparsity, bf16 bitmask format, decode M={args.m}", "M": args.m},
             "cpu_baseline": {"value": value, "unit": "tok/s", "cores": cores, "kind": "oracle",
                              "sample": f"each step: every {REF_ROW_FRACTION}th output row of the four layer-0 "
                                        f"linears at M={args.m}; time scaled x{REF_ROW_FRACTION * LAYERS}"},
@@ -448,13 +446,66 @@ def chain_parity(cs, M: int, oracle) -> dict:
             "what": "layer 0 of the chained step, each linear on the GPU's own inputs vs the float64 oracle"}
 
 
-def per_linear_section(args, Ms, world, dev, peak_gbs):
-    """Each shape's 32 layers as separate sp_linear launches (one CUDA graph per shape),
-    with the bench's own seeded N(0, 0.02^2) weights; per-launch times per shape."""
+def chained_section(args, peak_gbs, host_bf):
+    """The decode step of the 32-layer linear stack with its elementwise glue (residual adds,
+    gate*up), bf16 70%, run two ways on the same weights: one sp_chain_run launch per step
+    (glue fused into the epilogues) and a CUDA graph of separate launches (sp_linear plus
+    the glue kernels).  Parity of the chained launch: layer 0, linear by linear, against the
+    float64 oracle on the GPU's own inputs."""
     import torch
 
-    from paper_2405_03594_gb300 import sp
+    from paper_2405_03594_gb300 import sp, synth
+    from paper_2405_03594_gb300.stack import ChainStack, LinearStack
 
+    out = {"workload": f"llama2-7b linear stack decode step, {LAYERS} layers x (qkv, o + residual, gate_up -> "
+                       f"gate*up, down + residual), {args.pct}% bf16, N(0, 0.003^2) weights",
+           "chain": {}, "graph": {}}
+    cs = ChainStack(layers=LAYERS, pct=args.pct, int8=False, max_m=4, host=host_bf)
+    for M in (1, 4):
+        ms, cu = time_chain(cs, M, max(3, min(args.steps, 100)), max(3, args.warmup), 1)
+        b = chain_bytes(cs, M)
+        out["chain"][str(M)] = {"tok_s": M / (ms * 1e-3), "ms_per_step": ms, "chain_us": cu,
+                                "gbs": b / (cu * 1e-6) / 1e9, "frac_of_peak": b / (cu * 1e-6) / 1e9 / peak_gbs,
+                                "launches_per_step": cs.launches_per_step(M), "kernel": "chain_kernel",
+                                "activations_finite": bool(torch.isfinite(cs.h[:M].float()).all().item())}
+    if not args.no_cpu:
+        import oracle
+
+        oracle.build()
+        x = synth.activations(1, 4096, synth.rng(0, 0, 0, synth.STREAM_X))
+        cs.set_input(torch.from_numpy(x.view(np.int16)).to(cs.dev).view(torch.bfloat16))
+        out["chain_parity_layer0_M1"] = chain_parity(cs, 1, oracle)
+    del cs
+    torch.cuda.empty_cache()
+    st = LinearStack(layers=LAYERS, pct=args.pct, int8=False, max_m=4, host=host_bf)
+    for M in (1, 4):
+        x = synth.activations(M, 4096, synth.rng(0, 0, 0, synth.STREAM_X))
+        st.set_input(torch.from_numpy(x.view(np.int16)).to(st.dev).view(torch.bfloat16))
+        g = st.capture(M)
+        ms = time_graph(g, max(3, min(args.steps, 100)), max(3, args.warmup))
+        sp.check()
+        out["graph"][str(M)] = {"tok_s": M / (ms * 1e-3), "ms_per_step": ms,
+                                "launches_per_step": st.launches_per_step(M)}
+        del g
+    del st
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    from paper_2405_03594_gb300 import sp, synth
+
+    Ms = sorted({args.m} | {int(v) for v in args.sweep.split(",") if v.strip()})
     Mmax = max(Ms)
     host = host_layer(args.pct, Mmax)
     mats, xs, ys = {}, {}, {}
@@ -469,11 +520,11 @@ def per_linear_section(args, Ms, world, dev, peak_gbs):
     ws_bytes = max(h.workspace_size(Mmax) for h in (mats[n][0] for n in SHAPES))
     ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
 
-    def linear(name, layer, M):
-        mats[name][layer].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path)
+    def linear(name, layer, M, stream=None):
+        mats[name][layer].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path, stream=stream)
 
-    results = {}
-    for M in Ms:
+    def per_m(M):
+        # one CUDA graph per shape: its 32 layers back to back
         for name in SHAPES:
             linear(name, 0, M)
         torch.cuda.synchronize()
@@ -486,169 +537,170 @@ def per_linear_section(args, Ms, world, dev, peak_gbs):
             graphs[name] = g
         torch.cuda.synchronize()
         stream = torch.cuda.current_stream()
-        steps = max(3, min(args.steps, 50))
-        for _ in range(max(3, args.warmup)):
+        for _ in range(args.warmup):
             for name in SHAPES:
                 graphs[name].replay()
         torch.cuda.synchronize()
         ev = {name: [] for name in SHAPES}
-        t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
         t_start.record(stream)
-        for _ in range(steps):
+        for _ in range(args.steps):
             for name in SHAPES:
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
                 a.record(stream)
                 graphs[name].replay()
                 b.record(stream)
                 ev[name].append((a, b))
         t_end.record(stream)
         torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        total_ms = t_start.elapsed_time(t_end)
+        shape_ms = {name: sum(a.elapsed_time(b) for a, b in ev[name]) for name in SHAPES}
         sp.check()
-        step_ms = t_start.elapsed_time(t_end) / steps
-        per_shape = {}
+        return total_ms, shape_ms, graphs
+
+    results = {}
+    peak_gbs, peak_kind = load_peaks()
+    for M in Ms:
+        if M == args.m:
+            with ClockSampler(local_rank) as clk:
+                total_ms, shape_ms, graphs = per_m(M)
+            clocks = clk.summary()
+        else:
+            total_ms, shape_ms, graphs = per_m(M)
+        del graphs
+        step_ms = total_ms / args.steps
+        if world > 1:
+            t = torch.tensor([step_ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            step_ms = float(t.item())
         step_bytes = 0
+        per_shape = {}
         for name in SHAPES:
             h = mats[name][0]
             b = algorithmic_bytes(h.info, M, h.k, h.n)
             step_bytes += LAYERS * b
-            us = sum(a.elapsed_time(e) for a, e in ev[name]) / (steps * LAYERS) * 1e3
-            per_shape[name] = {"us": round(us, 3), "gbs": round(b / (us * 1e-6) / 1e9, 1),
-                               "frac": round(b / (us * 1e-6) / 1e9 / peak_gbs, 4),
-                               "kernel": h.kernel_name(M, args.path), "launches": h.launch_count(M, args.path)}
-        results[str(M)] = {"tok_s": world * M / (step_ms * 1e-3), "step_ms": step_ms,
-                           "step_gbs": step_bytes / (step_ms * 1e-3) / 1e9,
-                           "frac_of_peak": step_bytes / (step_ms * 1e-3) / 1e9 / peak_gbs, "per_shape": per_shape}
-        del graphs
-    out = {"workload": f"each shape's {LAYERS} layers as separate launches (one CUDA graph per shape), "
-                       f"{args.pct}% bf16, N(0, 0.02^2) weights", "per_m": results}
-    del mats
-    torch.cuda.empty_cache()
-    return out
-
-
-def run_ours(args):
-    import torch
-
-    rank, local_rank, world = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    from paper_2405_03594_gb300 import sp, synth
-    from paper_2405_03594_gb300.stack import ChainStack, host_layer as stack_host_layer
+            launch_us = shape_ms[name] / (args.steps * LAYERS) * 1e3
+            per_shape[name] = {"us_per_launch": launch_us, "algorithmic_bytes": b,
+                               "gbs": b / (launch_us * 1e-6) / 1e9, "frac": b / (launch_us * 1e-6) / 1e9 / peak_gbs}
+        results[M] = {"step_ms": step_ms, "tok_s": world * M / (step_ms * 1e-3),
+                      "step_gbs": step_bytes / (step_ms * 1e-3) / 1e9, "per_shape": per_shape,
+                      "step_bytes": step_bytes}
 
     M = args.m
-    if not 1 <= M <= 4:
-        raise SystemExit("the decode-step bench runs the chained kernel: --m must be 1..4")
-    peak_gbs, peak_kind = load_peaks()
-    sweep = sorted({int(v) for v in args.sweep.split(",") if v.strip()})
-
-    # ---------------------------------------------------------------- headline: chained decode step
-    host_bf = stack_host_layer(args.pct, False)
-    cs = ChainStack(layers=LAYERS, pct=args.pct, int8=False, max_m=4, host=host_bf)
-    with ClockSampler(local_rank) as clk:
-        step_ms, chain_us = time_chain(cs, M, args.steps, args.warmup, world)
-    clocks = clk.summary()
-    if world > 1:
-        t = torch.tensor([step_ms, chain_us], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        step_ms, chain_us = float(t[0].item()), float(t[1].item())
-    bytes_launch = chain_bytes(cs, M)
-    achieved = bytes_launch / (chain_us * 1e-6) / 1e9
-    workload = f"chain {LAYERS}x4 linears {args.pct}% bf16 M={M}"
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak_gbs, "unit": "GB/s", "frac": achieved / peak_gbs,
-                "traffic": profiled_traffic("chain_kernel", workload), "kernel": "chain_kernel", "launch": workload,
+    r = results[M]
+    dom = max(SHAPES, key=lambda n: r["per_shape"][n]["us_per_launch"])
+    d = r["per_shape"][dom]
+    kern = mats[dom][0].kernel_name(M, args.path)
+    workload = f"{dom} {args.pct}% bf16 M={M}"
+    roofline = {"bound": "hbm", "achieved": d["gbs"], "peak": peak_gbs, "unit": "GB/s", "frac": d["frac"],
+                "traffic": profiled_traffic(kern, workload), "kernel": kern, "launch": workload,
                 "peak_kind": f"of {peak_kind} (MEASURED_PEAKS.json hbm_gbs, copy)" if peak_kind == "measured"
                 else "of fallback",
-                "algorithmic_bytes_per_launch": bytes_launch, "us_per_launch": chain_us}
-    chain_per_m = {str(M): {"tok_s": world * M / (step_ms * 1e-3), "step_ms": step_ms, "chain_us": chain_us,
-                            "gbs": achieved, "frac": achieved / peak_gbs}}
-    for m in sweep:
-        if m <= 4 and m != M:
-            sm, cu = time_chain(cs, m, max(3, min(args.steps, 50)), max(3, args.warmup), world)
-            bl = chain_bytes(cs, m)
-            chain_per_m[str(m)] = {"tok_s": world * m / (sm * 1e-3), "step_ms": sm, "chain_us": cu,
-                                   "gbs": bl / (cu * 1e-6) / 1e9, "frac": bl / (cu * 1e-6) / 1e9 / peak_gbs}
+                "algorithmic_bytes_per_launch": d["algorithmic_bytes"], "us_per_launch": d["us_per_launch"]}
 
-    # ---------------------------------------------------------------- end to end (public API, host copies)
-    pinned_x = torch.from_numpy(synth.activations(M, 4096, synth.rng(0, 0, 0, synth.STREAM_X)).view(np.int16)) \
-        .view(torch.bfloat16).pin_memory()
-    pinned_y = torch.empty((M, 4096), dtype=torch.bfloat16).pin_memory()
+    # ---------------------------------------------------------------- end to end
+    # Public API calls (no graph), inputs copied from pinned host memory every step and
+    # the step's result (the last down projection) copied back.
+    pinned_x = {name: xs[name][:M].cpu().pin_memory() for name in SHAPES}
+    pinned_y = torch.empty((M, mats["down"][0].n), dtype=torch.bfloat16).pin_memory()
     stream = torch.cuda.current_stream()
     e2e_steps = max(3, min(args.steps, 50))
 
     def e2e_step():
-        cs.x0[:M].copy_(pinned_x, non_blocking=True)
-        cs.step(M, reset=True)
-        pinned_y.copy_(cs.h[:M], non_blocking=True)
+        for name in SHAPES:
+            xs[name][:M].copy_(pinned_x[name], non_blocking=True)
+        for layer in range(LAYERS):
+            for name in SHAPES:
+                linear(name, layer, M)
+        pinned_y.copy_(ys["down"][:M], non_blocking=True)
 
     for _ in range(2):
         e2e_step()
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
     a.record(stream)
     for _ in range(e2e_steps):
         e2e_step()
     b.record(stream)
     torch.cuda.synchronize()
-    sp.check()
     e2e_ms = a.elapsed_time(b) / e2e_steps
     if world > 1:
         t = torch.tensor([e2e_ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         e2e_ms = float(t.item())
+    h2d = sum(pinned_x[n].numel() * 2 for n in SHAPES)
+    d2h = pinned_y.numel() * 2
 
     # ---------------------------------------------------------------- parity + CPU oracle (rank 0, N=1)
     cpu = None
     parity = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        import oracle
+        cpu, outs = cpu_oracle_leg(host, M)
+        worst = 0.0
+        fro = 0.0
+        for name in SHAPES:
+            mats[name][0].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path)
+            y = synth.bf16_to_f32(ys[name][:M].view(torch.int16).cpu().numpy().view(np.uint16)).astype(np.float64)
+            ref = outs[name]
+            worst = max(worst, float(np.abs(y - ref).max() / np.abs(ref).max()))
+            fro = max(fro, float(np.linalg.norm(y - ref) / np.linalg.norm(ref)))
+        parity = {"max_err_over_max_ref": worst, "rel_fro": fro, "ok": worst <= 1e-2 and fro <= 5e-3}
 
-        oracle.build()
-        parity = chain_parity(cs, M, oracle)
-        host3 = {name: (W, mask, synth.activations(M, W.shape[1], synth.rng(0, 0, 0, synth.STREAM_X)))
-                 for name, (W, mask, _) in host_bf.items()}
-        cpu, _ = cpu_oracle_leg(host3, M)
-    del cs
+    # kernel launches per linear of the timed step (the library's own count)
+    launch_counts = {name: mats[name][0].launch_count(M, args.path) for name in SHAPES}
+    del mats
     torch.cuda.empty_cache()
+    host_bf = None
+    if not (args.no_chain and args.no_stack):
+        from paper_2405_03594_gb300.stack import host_layer as stack_host_layer
 
-    per_linear = None if args.no_per_linear else per_linear_section(args, sorted(set(sweep) | {M}), world, dev,
-                                                                    peak_gbs)
-    stack = None if args.no_stack else stack_section(args, peak_gbs, host_bf)
+        host_bf = stack_host_layer(args.pct, False)
+    chained = None if (args.no_chain or world > 1) else chained_section(args, peak_gbs, host_bf)
+    stack = None if (args.no_stack or world > 1) else stack_section(args, peak_gbs, host_bf)
     prefill = None if (args.no_prefill or world > 1) else prefill_section(args)
 
     if rank == 0:
+        launches_per_step = LAYERS * sum(launch_counts.values())
         line = {
-            "metric": METRIC, "value": world * M / (step_ms * 1e-3), "unit": "tok/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic: seeded N(0,0.003^2) bf16 weights (the chained stack's scale), per-row magnitude "
-                    "masks, N(0,1) bf16 x; 32 device copies of layer 0",
-            "config": {"workload": f"llama2-7b decode step through the linear stack: {LAYERS} layers x (qkv "
-                                   f"4096->12288, o 4096->4096 + residual, gate_up 4096->22016 -> gate*up, down "
-                                   f"11008->4096 + residual), chained, {args.pct}% per-row magnitude sparsity, bf16 "
-                                   f"bitmask format, decode M={M}, one persistent launch per step",
-                       "M": M, "layers": LAYERS, "sparsity_pct": args.pct,
-                       "l2": f"no flush: inputs larger than L2 ({bytes_launch / 1e9:.2f} GB of distinct compressed "
-                             f"weights per step)",
+            "metric": METRIC, "value": r["tok_s"], "unit": "tok/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded N(0,0.02^2) bf16 weights, per-row magnitude masks, N(0,1) bf16 x; "
+                    "32 device copies of layer 0",
+            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
+                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
+                                   f"sparsity, bf16 bitmask format, decode M={M}",
+                       "M": M, "layers": LAYERS, "sparsity_pct": args.pct, "path": args.path,
+                       "l2": f"no flush: inputs larger than L2 ({r['step_bytes'] / 1e9:.2f} GB of distinct "
+                             f"compressed weights per step)",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
-            "e2e": {"value": world * M / (e2e_ms * 1e-3), "unit": "tok/s", "h2d_bytes_per_step": pinned_x.numel() * 2,
-                    "d2h_bytes_per_step": pinned_y.numel() * 2,
-                    "how": "public API per step (x copied in from pinned host memory, sp_copy_columns + sp_chain_run, "
-                           "h copied out), no graph"},
-            "gpu_launches": 2 * args.steps,
+            "e2e": {"value": world * M / (e2e_ms * 1e-3), "unit": "tok/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "how": "public sp.linear calls (no graph) with pinned host x "
+                                                      "copied in and the last down output copied out per step"},
+            "gpu_launches": launches_per_step * args.steps,
             "roofline": roofline,
             "cpu_baseline": cpu,
             "clocks": clocks,
+            "step_gbs": r["step_gbs"],
             "parity_layer0": parity,
-            "chain_per_m": chain_per_m,
-            "per_linear": per_linear,
+            "chained_step_bf16": chained,
             "stack_int8": stack,
             "prefill": prefill,
+            "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
+                               "frac_of_peak": v["step_gbs"] / peak_gbs,
+                               "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),
+                                                 "frac": round(s["frac"], 4)} for n, s in v["per_shape"].items()}}
+                      for m, v in results.items()},
         }
         print(json.dumps(line), flush=True)
     if world > 1:
