@@ -81,6 +81,24 @@ def algorithmic_bytes(info, M: int, K: int, N: int) -> int:
     return int(info.nnz) * esize + N * K // 8 + int(info.scale_bytes) + 2 * M * K + 2 * M * N
 
 
+def max_over_ranks(vals, device=None):
+    """Element-wise maximum of `vals` over all ranks of the process group (the slowest
+    replica sets the step time); the values themselves with one process."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in vals]
+    t = torch.tensor([float(v) for v in vals], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def whole_job_tok_s(world: int, M: int, step_ms: float) -> float:
+    """Tokens per second of all replicas together: every rank decodes M tokens per step."""
+    return world * M / (step_ms * 1e-3)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -575,11 +593,7 @@ def run_ours(args):
         else:
             total_ms, shape_ms, graphs = per_m(M)
         del graphs
-        step_ms = total_ms / args.steps
-        if world > 1:
-            t = torch.tensor([step_ms], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            step_ms = float(t.item())
+        step_ms = max_over_ranks([total_ms / args.steps], dev)[0]
         step_bytes = 0
         per_shape = {}
         for name in SHAPES:
@@ -589,7 +603,7 @@ def run_ours(args):
             launch_us = shape_ms[name] / (args.steps * LAYERS) * 1e3
             per_shape[name] = {"us_per_launch": launch_us, "algorithmic_bytes": b,
                                "gbs": b / (launch_us * 1e-6) / 1e9, "frac": b / (launch_us * 1e-6) / 1e9 / peak_gbs}
-        results[M] = {"step_ms": step_ms, "tok_s": world * M / (step_ms * 1e-3),
+        results[M] = {"step_ms": step_ms, "tok_s": whole_job_tok_s(world, M, step_ms),
                       "step_gbs": step_bytes / (step_ms * 1e-3) / 1e9, "per_shape": per_shape,
                       "step_bytes": step_bytes}
 
@@ -633,11 +647,7 @@ def run_ours(args):
         e2e_step()
     b.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = a.elapsed_time(b) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks([a.elapsed_time(b) / e2e_steps], dev)[0]
     h2d = sum(pinned_x[n].numel() * 2 for n in SHAPES)
     d2h = pinned_y.numel() * 2
 
@@ -684,7 +694,7 @@ def run_ours(args):
                        "l2": f"no flush: inputs larger than L2 ({r['step_bytes'] / 1e9:.2f} GB of distinct "
                              f"compressed weights per step)",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
-            "e2e": {"value": world * M / (e2e_ms * 1e-3), "unit": "tok/s", "h2d_bytes_per_step": h2d,
+            "e2e": {"value": whole_job_tok_s(world, M, e2e_ms), "unit": "tok/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "how": "public sp.linear calls (no graph) with pinned host x "
                                                       "copied in and the last down output copied out per step"},
             "gpu_launches": launches_per_step * args.steps,
