@@ -542,7 +542,7 @@ def run_ours(args):
         mats[name][layer].linear(xs[name][:M], out=ys[name][:M], workspace=ws, path=args.path, stream=stream)
 
     def per_m(M):
-        # one CUDA graph per shape: its 32 layers back to back
+        # per-launch times: one CUDA graph per shape, its 32 layers back to back
         for name in SHAPES:
             linear(name, 0, M)
         torch.cuda.synchronize()
@@ -578,9 +578,31 @@ def run_ours(args):
         torch.cuda.synchronize()
         if world > 1:
             torch.distributed.barrier()
-        total_ms = t_start.elapsed_time(t_end)
         shape_ms = {name: sum(a.elapsed_time(b) for a, b in ev[name]) for name in SHAPES}
         sp.check()
+        # the decode step itself: the 128 linears in layer order (qkv, o, gate_up, down of
+        # layer 0, then layer 1, ...) in one graph; its time is the step time
+        gs = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gs):
+            for layer in range(LAYERS):
+                for name in SHAPES:
+                    linear(name, layer, M)
+        for _ in range(args.warmup):
+            gs.replay()
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+        t_start.record(stream)
+        for _ in range(args.steps):
+            gs.replay()
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        total_ms = t_start.elapsed_time(t_end)
+        sp.check()
+        graphs["step"] = gs
         return total_ms, shape_ms, graphs
 
     results = {}
