@@ -295,3 +295,41 @@ def test_chain_argument_errors():
     c.m = 0
     c.run()
     sp.check()
+
+
+def test_chain_longer_than_one_launch(oracle):
+    """164 linears (41 small layers): sp_chain_run splits them into launches of at most 160;
+    the linears on both sides of the split are checked from the GPU's own state, so the
+    second launch must see everything the first one wrote."""
+    from paper_2405_03594_gb300 import sp
+
+    M = 2
+    st = MiniStack(D=64, F=96, layers=41, pct=70, int8=False, std=0.02, seed=5)
+    ops = st.ops(M)
+    assert len(ops) == 164
+    x0 = synth.activations(M, 64, synth.rng(4, 0, 0, synth.STREAM_X))
+
+    def state_after(k):
+        st.reset(x0)
+        if k:
+            sp.Chain([o for _, _, o in ops[:k]], M).run()
+            sp.check()
+        return st.state(M)
+
+    prev = state_after(158)
+    for k in (159, 160, 161, 162):
+        cur = state_after(k)
+        name, l, _ = ops[k - 1]
+        host = st.host[l][name]
+        what = f"linear {k - 1} ({name}, layer {l})"
+        if name == "qkv":
+            gu.assert_close(_f(cur["qkv"]), _lin(oracle, host, prev["h"]), what)
+        elif name in ("o", "down"):
+            xin = prev["qkv"][:, 2 * st.D:] if name == "o" else prev["a"]
+            r = _f(st.r_host[2 * l + (0 if name == "o" else 1)])
+            ref = _f(prev["h"]) + _lin(oracle, host, np.ascontiguousarray(xin)) + r
+            gu.assert_close(_f(cur["h"]), ref, what)
+        else:
+            y = _lin(oracle, host, prev["h"])
+            gu.assert_close(_f(cur["a"]), y[:, 0::2] * y[:, 1::2], what)
+        prev = cur
