@@ -52,6 +52,7 @@ def parse():
     ap.add_argument("--no-stack", action="store_true", help="skip the INT8 32-layer stack section")
     ap.add_argument("--no-chain", action="store_true", help="skip the chained-step (glue included) section")
     ap.add_argument("--layers", type=int, default=32, help="profiling aid (--single chain): layers in the chain")
+    ap.add_argument("--int8", action="store_true", help="profiling aid (--single <shape>): INT8 values + fp32 scales")
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
                     help="profiling aid: time one layer-0 linear of this shape, or the chained step of --layers "
@@ -759,7 +760,12 @@ def run_single(args):
 
     dev = torch.device("cuda", 0)
     W, mask, x = synth.layer_inputs(args.single, args.pct, args.m, seed=0, layer=0)
-    h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16), torch.from_numpy(mask).to(dev))
+    if args.int8:
+        q, sc = synth.quantize_int8(W, mask)
+        h = sp.compress(torch.from_numpy(q).to(dev), torch.from_numpy(mask).to(dev), torch.from_numpy(sc).to(dev))
+    else:
+        h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
+                        torch.from_numpy(mask).to(dev))
     xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
     y = torch.empty((args.m, h.n), dtype=torch.bfloat16, device=dev)
     ws = torch.zeros(max(h.workspace_size(args.m), 256), dtype=torch.uint8, device=dev)
@@ -775,7 +781,7 @@ def run_single(args):
     sp.check()
     us = a.elapsed_time(b) / max(args.steps, 1) * 1e3
     nbytes = algorithmic_bytes(h.info, args.m, h.k, h.n)
-    print(json.dumps({"single": args.single, "M": args.m, "pct": args.pct, "us_per_launch": us,
+    print(json.dumps({"single": args.single, "M": args.m, "pct": args.pct, "int8": args.int8, "us_per_launch": us,
                       "algorithmic_bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}), flush=True)
 
 
