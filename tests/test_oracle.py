@@ -244,6 +244,37 @@ def test_int8_oracle_integer_exact_and_scale(oracle):
     assert np.array_equal(oracle.linear_from_format(buf, off, N, K, 1, x, s), ys)
 
 
+# ---------------------------------------------------------------- stack glue
+
+# bf16 bit patterns of exactly representable values (sign, 8-bit exponent, 7-bit mantissa):
+# 1.0 = 0x3F80, 1.5 = 0x3FC0, -0.25 = 0xBE80, 2.0 = 0x4000, -3.0 = 0xC040, 10.0 = 0x4120,
+# 0.125 = 0x3E00, 0.5 = 0x3F00, 4.0 = 0x4080, -1.0 = 0xBF80.
+_BF = {1.0: 0x3F80, 1.5: 0x3FC0, -0.25: 0xBE80, 2.0: 0x4000, -3.0: 0xC040, 10.0: 0x4120,
+       0.125: 0x3E00, 0.5: 0x3F00, 4.0: 0x4080, -1.0: 0xBF80}
+
+
+def _bits(rows):
+    return np.array([[_BF[v] for v in row] for row in rows], dtype=np.uint16)
+
+
+def test_bf16_bit_patterns_are_the_values():
+    for v, b in _BF.items():
+        assert np.array([b << 16], dtype=np.uint32).view(np.float32)[0] == v
+
+
+def test_glue_hand_derived_values(oracle):
+    """Residual add h + a + r with r broadcast over the rows, and the gate/up product of a
+    row laid out as [gate_0 .. gate_{F-1}, up_0 .. up_{F-1}]; expected values by hand."""
+    h = _bits([[1.5, -0.25, 2.0], [1.0, -3.0, 10.0]])
+    a = _bits([[2.0, 1.0, 0.125], [-0.25, 1.5, -3.0]])
+    r = _bits([[10.0, 0.125, -1.0]])[0]
+    out = oracle.residual_add(h, a, r)
+    assert np.array_equal(out, np.array([[13.5, 0.875, 1.125], [10.75, -1.375, 6.0]]))
+    g = _bits([[1.5, -0.25, 2.0, 4.0], [-3.0, 0.5, 10.0, 0.125]])
+    out = oracle.mul_halves(g)
+    assert np.array_equal(out, np.array([[3.0, -1.0], [-30.0, 0.0625]]))
+
+
 # ---------------------------------------------------------------- input generator
 
 

@@ -23,6 +23,10 @@ MUTANTS = {
     "int8_scale_dropped": ("acc += or_bf16_to_double(x[m * K + k]) * ((double)q[n * K + k] * sn);",
                            "acc += or_bf16_to_double(x[m * K + k]) * ((double)q[n * K + k]);"),
     "block_mask_msb_first": ("m |= (uint64_t)1 << i;", "m |= (uint64_t)1 << (n - 1 - i);"),
+    "residual_r_dropped": (" + or_bf16_to_double(a[m * N + j]) + or_bf16_to_double(r[j]);",
+                           " + or_bf16_to_double(a[m * N + j]);"),
+    "halves_row_stride": ("or_bf16_to_double(g[m * 2 * F + j]) * or_bf16_to_double(g[m * 2 * F + F + j])",
+                          "or_bf16_to_double(g[m * F + j]) * or_bf16_to_double(g[m * F + F + j])"),
     "bf16_shift": ("uint32_t u = (uint32_t)h << 16;", "uint32_t u = (uint32_t)h << 15;"),
     "tile_width_off_by_one": ("for (int j = 0; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals",
                               "for (int j = 1; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals"),
@@ -43,6 +47,7 @@ def _pin_suite(o):
         "library_matmul": lambda: pins.test_linear_matches_float64_library_matmul(o, 70),
         "one_hot": lambda: pins.test_linear_one_hot_selects_a_column(o),
         "int8_exact": lambda: pins.test_int8_oracle_integer_exact_and_scale(o),
+        "glue": lambda: pins.test_glue_hand_derived_values(o),
     }
     failed = []
     for name, fn in checks.items():
