@@ -160,7 +160,9 @@ sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* 
  *   wrong results; order them on one stream. */
 sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* stream);
 
-/* A copy of the handle with its own device buffers (same bytes). */
+/* A copy of the handle with its own device buffers (same bytes), allocated on the
+ * current device, which must be the handle's (SP_ERR_INVALID_ARG otherwise).  The copies
+ * run on `stream`, which is synchronised before the call returns. */
 sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx, void* stream,
                    sp_matrix** out);
 

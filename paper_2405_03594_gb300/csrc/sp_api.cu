@@ -164,6 +164,12 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
   *out = nullptr;
   if (!live(h)) return SP_ERR_BAD_HANDLE;
   if ((alloc == nullptr) != (free_fn == nullptr)) return SP_ERR_INVALID_ARG;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
+  if (dev != h->device) return SP_ERR_INVALID_ARG;  // the copy lives on the source's device
   sp_matrix* c = new sp_matrix(*h);
   c->magic = 0;
   c->alloc = alloc;
@@ -192,6 +198,8 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
     st = SP_ERR_CUDA;
   }
   if (st != SP_OK) {
+    cudaGetLastError();
+    cudaStreamSynchronize(s);  // no copy may still target the buffers handed back below
     cudaGetLastError();
     dev_free(c, c->d_buf);
     dev_free(c, c->d_off);

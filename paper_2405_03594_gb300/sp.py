@@ -130,7 +130,12 @@ def _ptr(t: torch.Tensor | None) -> ctypes.c_void_p:
 
 
 class SparseMatrix:
-    """A compressed weight owned by libsp (the handle) with torch-allocated buffers."""
+    """A compressed weight owned by libsp (the handle) with torch-allocated buffers.
+
+    The buffers come from PyTorch's caching allocator on the stream that was current at
+    compression, so, as for any torch tensor, their reuse after release is ordered on that
+    stream only: work queued on other streams must be complete before the handle is
+    dropped (free() synchronises the device first; garbage collection does not)."""
 
     def __init__(self, handle: ctypes.c_void_p):
         self._h = handle
