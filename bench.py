@@ -23,6 +23,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import subprocess
 import sys
 import tempfile
@@ -221,13 +222,31 @@ def prefill_section(args):
     return res
 
 
-def kernel_source_hash():
+# The source files that compile into each profiled kernel (its translation unit and the
+# device headers it includes, plus the public headers without their comments); host-only
+# files such as sp_api.cu do not change the kernel.
+KERNEL_SOURCES = {
+    "linear_ccw_kernel": ("sp_linear_cc.cu", "sp_cc_common.cuh", "sp_internal.cuh"),
+    "linear_cc_kernel": ("sp_linear_cc.cu", "sp_cc_common.cuh", "sp_internal.cuh"),
+    "linear_tc_kernel": ("sp_linear_tc.cu", "sp_internal.cuh"),
+    "chain_kernel": ("sp_chain.cu", "sp_cc_common.cuh", "sp_internal.cuh"),
+}
+
+
+def kernel_source_hash(kernel: str):
+    """Hash of the sources of `kernel`; None for a kernel without a source list."""
+    files = KERNEL_SOURCES.get(kernel)
+    if files is None:
+        return None
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2405_03594_gb300", "csrc")
-    for n in sorted(os.listdir(csrc)):
-        if n.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, n), "rb") as f:
-                h.update(f.read())
+    for n in files:
+        with open(os.path.join(csrc, n), "rb") as f:
+            h.update(n.encode() + b"\0" + f.read())
+    for n in ("sp.h", "sp_stack.h"):
+        with open(os.path.join(ROOT, "include", n)) as f:
+            code = re.sub(r"/\*.*?\*/|//[^\n]*", "", f.read(), flags=re.S)
+        h.update(n.encode() + b"\0" + " ".join(code.split()).encode())
     return h.hexdigest()[:16]
 
 
@@ -240,7 +259,7 @@ def profiled_traffic(kernel: str, workload: str):
     with open(p) as f:
         d = json.load(f)
     e = d.get(f"{kernel}|{workload}")
-    if not e or e.get("source_hash") != kernel_source_hash():
+    if not e or e.get("source_hash") is None or e.get("source_hash") != kernel_source_hash(kernel):
         return None
     return e.get("dram_bytes_per_launch")
 

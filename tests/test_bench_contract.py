@@ -41,3 +41,54 @@ def test_our_arm_fails_loudly_without_a_gpu():
     p = _run("--steps", "1", "--warmup", "3", timeout=300)
     assert p.returncode != 0
     assert not [ln for ln in p.stdout.splitlines() if ln.startswith("{")]
+
+
+def _bench_module():
+    import importlib.util
+
+    spec = importlib.util.spec_from_file_location("bench_under_test", os.path.join(ROOT, "bench.py"))
+    b = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(b)
+    return b
+
+
+def test_traffic_staleness_hash_follows_the_kernel_sources(tmp_path):
+    """The committed ncu traffic stays valid across host-only edits and comment edits of
+    the public headers, and is dropped once a source of the kernel itself changes."""
+    import shutil
+
+    b = _bench_module()
+    for d in ("paper_2405_03594_gb300/csrc", "include"):
+        shutil.copytree(os.path.join(ROOT, d), tmp_path / d)
+    b.ROOT = str(tmp_path)
+    base = {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES}
+    assert b.kernel_source_hash("no_such_kernel") is None
+
+    def edit(rel, old, new):
+        p = tmp_path / rel
+        s = p.read_text()
+        assert old in s
+        p.write_text(s.replace(old, new, 1))
+
+    edit("paper_2405_03594_gb300/csrc/sp_api.cu", "extern \"C\" {", "extern \"C\" {\n// host-only edit")
+    edit("include/sp.h", "/*", "/* comment edit;")
+    assert {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES} == base
+    edit("paper_2405_03594_gb300/csrc/sp_linear_tc.cu", "namespace sp {", "namespace sp {\nstatic int edited;")
+    now = {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES}
+    assert now["linear_tc_kernel"] != base["linear_tc_kernel"]
+    assert all(now[k] == base[k] for k in base if k != "linear_tc_kernel")
+    edit("include/sp.h", "#define", "#define SP_EDITED 1\n#define")
+    assert all(b.kernel_source_hash(k) != base[k] for k in base)
+
+
+def test_committed_traffic_matches_the_current_kernel_sources():
+    """Each committed ncu traffic figure carries the hash of the sources it was taken on;
+    those that still match the current sources are the ones the bench reports."""
+    b = _bench_module()
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        d = json.load(f)
+    for key, e in d.items():
+        kernel, workload = key.split("|", 1)
+        assert kernel in b.KERNEL_SOURCES and e["dram_bytes_per_launch"] > 0
+        got = b.profiled_traffic(kernel, workload)
+        assert got == (e["dram_bytes_per_launch"] if e["source_hash"] == b.kernel_source_hash(kernel) else None)
