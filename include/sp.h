@@ -106,10 +106,13 @@ sp_status sp_compress(const void* w_dev, const uint8_t* mask_dev, int64_t n, int
                       void* stream, sp_matrix** out);
 
 /* Expand the handle back to the dense masked weight: w_out_dev [N, K] of the
- * handle's dtype, zero where masked out, bit-exact. */
+ * handle's dtype (int8 values without their scales for SP_INT8), zero where masked
+ * out, bit-exact.  Asynchronous on `stream`; w_out_dev is caller-owned.
+ * SP_ERR_BAD_HANDLE for a dead handle, SP_ERR_INVALID_ARG for a null output. */
 sp_status sp_decompress(const sp_matrix* h, void* w_out_dev, void* stream);
 
-/* Bytes of device workspace that sp_linear needs for a batch of m rows (may be 0). */
+/* Bytes of device workspace that sp_linear needs for a batch of m rows, written to
+ * *bytes (0 for m == 0).  Host only.  SP_ERR_INVALID_ARG for m < 0 or a null `bytes`. */
 sp_status sp_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
 
 /* y = x . (W o Mask)^T, FP32 accumulation, bf16 output (round to nearest even).
@@ -170,6 +173,9 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
  * work still reads them (e.g. synchronise the stream first).  NULL is a no-op. */
 sp_status sp_free(sp_matrix* h);
 
+/* Shape and storage facts of a live handle, written to *info (the fields of sp_info_t).
+ * Host only, no GPU work.  SP_ERR_BAD_HANDLE for a dead handle, SP_ERR_INVALID_ARG for a
+ * null `info`. */
 sp_status sp_info(const sp_matrix* h, sp_info_t* info);
 
 /* Synchronously copy the compressed bytes (info.bytes) and the RB*T+1 chunk
