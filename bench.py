@@ -317,8 +317,9 @@ class ClockSampler:
 
 
 def cpu_oracle_leg(host, M: int, reps_target_s: float = 10.0):
-    """Time the float64 oracle on this host's cores on layer 0 (all four linears) and
-    scale to a 32-layer step.  Returns (cpu_baseline dict, oracle outputs)."""
+    """Time the float64 oracle on this host's cores on layer 0 (all four linears),
+    repeated for about `reps_target_s` seconds (at least three runs), and scale the median
+    run to a 32-layer step.  Returns (cpu_baseline dict, oracle outputs)."""
     cores = len(os.sched_getaffinity(0))
     os.environ.setdefault("OMP_NUM_THREADS", str(cores))
     import oracle
@@ -332,7 +333,7 @@ def cpu_oracle_leg(host, M: int, reps_target_s: float = 10.0):
             W, mask, x = host[name]
             outs[name] = oracle.linear_bf16(x[:M], W, mask)
         t_layer.append(time.perf_counter() - t0)
-        if time.perf_counter() > deadline or len(t_layer) >= 5:
+        if time.perf_counter() > deadline and len(t_layer) >= 3:
             break
     t = sorted(t_layer)[len(t_layer) // 2]
     return ({"value": M / (LAYERS * t), "unit": "tok/s", "cores": cores, "kind": "oracle",

@@ -92,3 +92,29 @@ def test_committed_traffic_matches_the_current_kernel_sources():
         assert kernel in b.KERNEL_SOURCES and e["dram_bytes_per_launch"] > 0
         got = b.profiled_traffic(kernel, workload)
         assert got == (e["dram_bytes_per_launch"] if e["source_hash"] == b.kernel_source_hash(kernel) else None)
+
+
+def test_cpu_baseline_leg_runs_the_oracle_for_the_requested_time():
+    """The bench's cpu_baseline: the float64 oracle on the host cores, repeated for about
+    the requested time (at least three runs), scaled to a full step."""
+    import time
+
+    import numpy as np
+
+    b = _bench_module()
+    g = np.random.default_rng(0)
+    host = {}
+    for name in b.SHAPES:
+        N, K = 40, 64
+        W = g.standard_normal((N, K)).astype(np.float32)
+        host[name] = (b.np.asarray(W.view(np.uint32) >> 16, dtype=np.uint16),
+                      (g.random((N, K)) < 0.3).astype(np.uint8),
+                      np.zeros((2, K), dtype=np.uint16))
+    t0 = time.perf_counter()
+    cb, outs = b.cpu_oracle_leg(host, 1, reps_target_s=0.3)
+    assert time.perf_counter() - t0 >= 0.3
+    assert cb["kind"] == "oracle" and cb["unit"] == "tok/s" and cb["cores"] >= 1 and cb["value"] > 0
+    runs = int(cb["sample"].split("median of ")[1].split()[0])
+    assert runs >= 3
+    assert set(outs) == set(b.SHAPES) and all(outs[n].shape == (1, 40) for n in b.SHAPES)
+    assert all(not outs[n].any() for n in b.SHAPES)  # x = 0 gives y = 0
