@@ -118,3 +118,12 @@ def test_cpu_baseline_leg_runs_the_oracle_for_the_requested_time():
     assert runs >= 3
     assert set(outs) == set(b.SHAPES) and all(outs[n].shape == (1, 40) for n in b.SHAPES)
     assert all(not outs[n].any() for n in b.SHAPES)  # x = 0 gives y = 0
+
+
+def test_dense_section_reports_failures_instead_of_raising():
+    """The dense cuBLAS comparison is context: on a host without a GPU it returns its
+    failure inside the section (with the paper's quoted speedups) rather than raising."""
+    b = _bench_module()
+    out = b.dense_section({}, {}, {}, [1])
+    assert "error" in out and out["paper"]["gpu_sparsity_only"]["x"] == 1.7
+    assert out["shapes"] == {} and out["step_speedup"] == {}
