@@ -31,7 +31,7 @@ def build(force: bool = False) -> str:
     """Compile sp_oracle.c into libsp_oracle.so next to it (gcc, -O2, OpenMP)."""
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".tmp{os.getpid()}"
-        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", _SRC, "-o", tmp])
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -52,6 +52,8 @@ def _bind(lib):
     lib.or_linear_from_format.restype = ctypes.c_int
     lib.or_residual_add.argtypes = [P, P, P, I64, I64, P]
     lib.or_mul_halves.argtypes = [P, I64, I64, P]
+    lib.or_masked_update_bf16.argtypes = [P, P, I64, I64, P, ctypes.c_float]
+    lib.or_masked_update_bf16.restype = ctypes.c_int
     lib.or_block_encode.argtypes = [P, ctypes.c_int, P, P]
     lib.or_block_encode.restype = ctypes.c_int
     return lib
@@ -179,4 +181,17 @@ def mul_halves(g: np.ndarray) -> np.ndarray:
     M, F2 = g.shape
     out = np.zeros((M, F2 // 2), dtype=np.float64)
     _load().or_mul_halves(_p(g), M, F2 // 2, _p(out))
+    return out
+
+
+def masked_update_bf16(buf: np.ndarray, off: np.ndarray, N: int, K: int, grad: np.ndarray, lr: float) -> np.ndarray:
+    """Algorithm 1's masked step on a compressed bf16 matrix: a copy of `buf` with every
+    kept value w replaced by bf16_rne(fmaf(-lr, grad, w)); grad is dense [N, K] float32."""
+    out = np.array(buf, dtype=np.uint8, copy=True)
+    off = np.ascontiguousarray(off, dtype=np.uint64)
+    g = np.ascontiguousarray(grad, dtype=np.float32)
+    assert g.shape == (N, K)
+    rc = _load().or_masked_update_bf16(_p(out), _p(off), N, K, _p(g), ctypes.c_float(lr))
+    if rc != 0:
+        raise ValueError("malformed compressed matrix")
     return out

@@ -33,9 +33,16 @@
  *    weights): the weight of row n is q[n,k] * s[n]; the oracle multiplies
  *    with exactly those quantized weights.
  *
+ *  - The masked weight update of sparse training (Sec. 2.1, Algorithm 1): the
+ *    gradient is multiplied by the fixed mask, the weights take one step of
+ *    size eta, and are multiplied by the mask again, so a pruned weight stays
+ *    zero.  On the compressed form only the kept entries exist, so the step
+ *    touches exactly the stored values; or_masked_update_bf16() applies it there.
+ *
  * Floating point: bf16 -> float32 -> double is exact; bf16 x bf16 and
  * bf16 x (int8 * fp32) products are exact in double; only the k-sum rounds.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -259,4 +266,49 @@ void or_mul_halves(const uint16_t* g, int64_t M, int64_t F, double* out) {
   for (int64_t m = 0; m < M; ++m)
     for (int64_t j = 0; j < F; ++j)
       out[m * F + j] = or_bf16_to_double(g[m * 2 * F + j]) * or_bf16_to_double(g[m * 2 * F + F + j]);
+}
+
+/* float32 -> bf16 bit pattern, round to nearest, ties to even (finite inputs): add just
+ * under half of the dropped 16-bit range, plus one when the kept part is odd, and drop
+ * the low half. */
+static uint16_t or_float_to_bf16_rne(float f) {
+  uint32_t u;
+  memcpy(&u, &f, sizeof u);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+/* The masked update of Algorithm 1 on the compressed form, bf16 values: for every kept
+ * (n, k), w[n,k] <- bf16(fmaf(-lr, grad[n,k], w[n,k])), one fused multiply-add in float32
+ * and one round to nearest even.  grad is dense [N, K] float32; its masked-out entries are
+ * never read.  The masks, offsets and padding do not change.  Updates buf in place;
+ * returns 0, or -1 for a mask bit outside the matrix. */
+int or_masked_update_bf16(uint8_t* buf, const uint64_t* off, int64_t N, int64_t K, const float* grad, float lr) {
+  int64_t T, RB;
+  or_geometry(N, K, &T, &RB);
+  for (int64_t rb = 0; rb < RB; ++rb) {
+    for (int64_t t = 0; t < T; ++t) {
+      uint8_t* chunk = buf + off[rb * T + t];
+      uint8_t* vals = chunk + OR_MASK_BYTES;
+      int64_t v = 0;
+      for (int r = 0; r < OR_CHUNK_ROWS; ++r) {
+        int64_t n = rb * OR_CHUNK_ROWS + r;
+        uint64_t m = or_read_u64le(chunk + r * 8);
+        for (int j = 0; j < OR_TILE_K; ++j) {
+          if (!((m >> j) & 1u)) continue;
+          int64_t k = t * OR_TILE_K + j;
+          if (n >= N || k >= K) return -1;
+          uint16_t h;
+          memcpy(&h, vals + v * 2, 2);
+          uint32_t u = (uint32_t)h << 16;
+          float w;
+          memcpy(&w, &u, sizeof w);
+          h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + k], w));
+          memcpy(vals + v * 2, &h, 2);
+          ++v;
+        }
+      }
+    }
+  }
+  return 0;
 }

@@ -275,6 +275,73 @@ def test_glue_hand_derived_values(oracle):
     assert np.array_equal(out, np.array([[3.0, -1.0], [-30.0, 0.0625]]))
 
 
+# ---------------------------------------------------------------- masked update (Sec. 2.1, Algorithm 1)
+
+
+def _one_entry_update(oracle, w_bits, g, lr):
+    """Compress a 3 x 72 matrix whose only kept entry is (1, 5) = w_bits, apply the masked
+    step with gradient g there (and 1e30 everywhere else), return the updated entry's bits."""
+    N, K = 3, 72
+    W = np.zeros((N, K), dtype=np.uint16)
+    W[1, 5] = w_bits
+    mask = np.zeros((N, K), dtype=np.uint8)
+    mask[1, 5] = 1
+    grad = np.full((N, K), 1e30, dtype=np.float32)
+    grad[1, 5] = g
+    buf, off = oracle.compress(W, mask)
+    out = oracle.masked_update_bf16(buf, off, N, K, grad, lr)
+    back = oracle.decompress(out, off, N, K, np.uint16)
+    assert not np.delete(back.ravel(), 1 * K + 5).any()
+    assert np.array_equal(out[:1024], buf[:1024]) and out.size == buf.size
+    return int(back[1, 5])
+
+
+def test_masked_update_hand_derived_rounding(oracle):
+    """w - lr*g rounded once to bf16, nearest-even: 1 + 2^-8 lies halfway between 1.0
+    (0x3F80, even) and 1 + 2^-7 (0x3F81); 1 + 3*2^-8 halfway between 0x3F81 and 0x3F82
+    (even); 1 + 2^-8 + 2^-20 just above halfway.  The other cases are exact."""
+    assert _one_entry_update(oracle, 0x3F80, -2.0 ** -8, 1.0) == 0x3F80
+    assert _one_entry_update(oracle, 0x3F80, -3 * 2.0 ** -8, 1.0) == 0x3F82
+    assert _one_entry_update(oracle, 0x3F80, -(2.0 ** -8 + 2.0 ** -20), 1.0) == 0x3F81
+    assert _one_entry_update(oracle, 0x4000, 4.0, 0.5) == 0x0000      # 2 - 0.5*4 = +0
+    assert _one_entry_update(oracle, 0xBFC0, 2.0, 0.25) == 0xC000     # -1.5 - 0.25*2 = -2
+    assert _one_entry_update(oracle, 0x3F80, 1.0, -1.0) == 0x4000     # 1 + 1 = 2 (negative step)
+
+
+def test_masked_update_equals_dense_step_then_compress(oracle):
+    """Algorithm 1 written densely: W' = bf16(W - lr * (grad o M)) o M, with the sum exact in
+    float64 (dyadic gradients with few bits), rounded to float32 and then to bf16 by torch;
+    compressing W' with the same mask must give the updated buffer byte for byte."""
+    import torch
+
+    N, K = 200, 136
+    W, mask, _ = _rand_case(N, K, 70, seed=11)
+    g = np.random.default_rng(12)
+    grad = (g.integers(-255, 256, size=(N, K)) * 2.0 ** -10).astype(np.float32)
+    lr = 2.0 ** -3
+    buf, off = oracle.compress(W, mask)
+    out = oracle.masked_update_bf16(buf, off, N, K, grad, lr)
+    w64 = synth.bf16_to_f32(W).astype(np.float64)
+    new32 = (w64 - lr * grad.astype(np.float64)).astype(np.float32)
+    new_bits = torch.from_numpy(new32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    expect_buf, expect_off = oracle.compress(np.where(mask != 0, new_bits, 0).astype(np.uint16), mask)
+    assert np.array_equal(expect_off, off)
+    assert np.array_equal(out, expect_buf)
+
+
+def test_masked_update_ignores_masked_out_gradient_and_zero_step(oracle):
+    N, K = 130, 72
+    W, mask, _ = _rand_case(N, K, 60, seed=13)
+    g = np.random.default_rng(14).standard_normal((N, K)).astype(np.float32)
+    buf, off = oracle.compress(W, mask)
+    noisy = np.where(mask != 0, g, np.float32(3e38)).astype(np.float32)
+    clean = np.where(mask != 0, g, np.float32(0)).astype(np.float32)
+    a = oracle.masked_update_bf16(buf, off, N, K, noisy, 0.01)
+    assert np.array_equal(a, oracle.masked_update_bf16(buf, off, N, K, clean, 0.01))
+    assert not np.array_equal(a, buf)
+    assert np.array_equal(oracle.masked_update_bf16(buf, off, N, K, noisy, 0.0), buf)
+
+
 # ---------------------------------------------------------------- input generator
 
 

@@ -27,6 +27,11 @@ MUTANTS = {
                            " + or_bf16_to_double(a[m * N + j]);"),
     "halves_row_stride": ("or_bf16_to_double(g[m * 2 * F + j]) * or_bf16_to_double(g[m * 2 * F + F + j])",
                           "or_bf16_to_double(g[m * F + j]) * or_bf16_to_double(g[m * F + F + j])"),
+    "update_sign": ("h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + k], w));",
+                    "h = or_float_to_bf16_rne(fmaf(lr, grad[n * K + k], w));"),
+    "update_truncates": ("u += 0x7FFFu + ((u >> 16) & 1u);", "u += 0u;"),
+    "update_grad_index": ("h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + k], w));",
+                          "h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + (k ^ 1)], w));"),
     "bf16_shift": ("uint32_t u = (uint32_t)h << 16;", "uint32_t u = (uint32_t)h << 15;"),
     "tile_width_off_by_one": ("for (int j = 0; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals",
                               "for (int j = 1; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals"),
@@ -48,6 +53,8 @@ def _pin_suite(o):
         "one_hot": lambda: pins.test_linear_one_hot_selects_a_column(o),
         "int8_exact": lambda: pins.test_int8_oracle_integer_exact_and_scale(o),
         "glue": lambda: pins.test_glue_hand_derived_values(o),
+        "update_rounding": lambda: pins.test_masked_update_hand_derived_rounding(o),
+        "update_dense": lambda: pins.test_masked_update_equals_dense_step_then_compress(o),
     }
     failed = []
     for name, fn in checks.items():
@@ -71,7 +78,7 @@ def test_each_planted_mistake_is_caught(oracle, tmp_path, name):
     path_c = tmp_path / "mut.c"
     path_c.write_text(mutated)
     so = tmp_path / "libmut.so"
-    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", str(path_c), "-o", str(so)])
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", str(path_c), "-o", str(so), "-lm"])
     oracle_mod.use_library(str(so))
     try:
         failed = _pin_suite(oracle_mod)
