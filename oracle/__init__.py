@@ -52,6 +52,7 @@ def _bind(lib):
     lib.or_linear_from_format.restype = ctypes.c_int
     lib.or_residual_add.argtypes = [P, P, P, I64, I64, P]
     lib.or_mul_halves.argtypes = [P, I64, I64, P]
+    lib.or_linear_w8a8.argtypes = [P, P, I64, P, P, P, I64, I64, P, P]
     lib.or_masked_update_bf16.argtypes = [P, P, I64, I64, P, ctypes.c_float]
     lib.or_masked_update_bf16.restype = ctypes.c_int
     lib.or_block_encode.argtypes = [P, ctypes.c_int, P, P]
@@ -136,6 +137,22 @@ def linear_int8(x: np.ndarray, q: np.ndarray, mask: np.ndarray, s: np.ndarray) -
     y = np.zeros((M, N), dtype=np.float64)
     _load().or_linear_int8(_p(x), M, _p(q), _p(mask), _p(s), N, K, _p(y))
     return y
+
+
+def linear_w8a8(qx: np.ndarray, sx: np.ndarray, qw: np.ndarray, mask: np.ndarray, sw: np.ndarray):
+    """INT8 weights and activations: (int64 acc [M, N], float64 y = sx[m] * sw[n] * acc)."""
+    qx = np.ascontiguousarray(qx, dtype=np.int8)
+    sx = np.ascontiguousarray(sx, dtype=np.float32)
+    qw = np.ascontiguousarray(qw, dtype=np.int8)
+    mask = np.ascontiguousarray(mask, dtype=np.uint8)
+    sw = np.ascontiguousarray(sw, dtype=np.float32)
+    M, K = qx.shape
+    N = qw.shape[0]
+    assert qw.shape == (N, K) and mask.shape == (N, K) and sx.shape == (M,) and sw.shape == (N,)
+    acc = np.zeros((M, N), dtype=np.int64)
+    y = np.zeros((M, N), dtype=np.float64)
+    _load().or_linear_w8a8(_p(qx), _p(sx), M, _p(qw), _p(mask), _p(sw), N, K, _p(acc), _p(y))
+    return acc, y
 
 
 def linear_from_format(buf, off, N: int, K: int, esize: int, x: np.ndarray, scale=None) -> np.ndarray:

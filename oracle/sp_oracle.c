@@ -33,6 +33,10 @@
  *    weights): the weight of row n is q[n,k] * s[n]; the oracle multiplies
  *    with exactly those quantized weights.
  *
+ *  - INT8 weights and INT8 activations (Sec. 3.4: the quantized sparse models
+ *    run with INT8 weights and activations): with per-token activation scales
+ *    sx[m] and per-row weight scales sw[n], y[m,n] = sx[m] * sw[n] *
+ *    sum_k qx[m,k] * qw[n,k] * Mask[n,k]; the integer sum is exact (int64).
  *  - The masked weight update of sparse training (Sec. 2.1, Algorithm 1): the
  *    gradient is multiplied by the fixed mask, the weights take one step of
  *    size eta, and are multiplied by the mask again, so a pruned weight stays
@@ -180,6 +184,22 @@ void or_linear_bf16(const uint16_t* x, int64_t M, const uint16_t* W, const uint8
       for (int64_t k = 0; k < K; ++k)
         if (mask[n * K + k]) acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);
       y[m * N + n] = acc;
+    }
+  }
+}
+
+/* INT8 weights and activations: acc[m,n] = sum_k qx[m,k] * qw[n,k] * Mask[n,k] exactly in
+ * int64, then y[m,n] = (sx[m] * sw[n]) * acc in float64 (the scale product is exact). */
+void or_linear_w8a8(const int8_t* qx, const float* sx, int64_t M, const int8_t* qw, const uint8_t* mask,
+                    const float* sw, int64_t N, int64_t K, int64_t* acc_out, double* y) {
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n) {
+    for (int64_t m = 0; m < M; ++m) {
+      int64_t acc = 0;
+      for (int64_t k = 0; k < K; ++k)
+        if (mask[n * K + k]) acc += (int64_t)qx[m * K + k] * (int64_t)qw[n * K + k];
+      if (acc_out) acc_out[m * N + n] = acc;
+      y[m * N + n] = ((double)sx[m] * (double)sw[n]) * (double)acc;
     }
   }
 }

@@ -275,6 +275,47 @@ def test_glue_hand_derived_values(oracle):
     assert np.array_equal(out, np.array([[3.0, -1.0], [-30.0, 0.0625]]))
 
 
+# ---------------------------------------------------------------- INT8 weights and activations (Sec. 3.4)
+
+
+def _w8a8_case(M, N, K, seed):
+    g = np.random.default_rng(seed)
+    qx = g.integers(-127, 128, size=(M, K)).astype(np.int8)
+    qw = g.integers(-127, 128, size=(N, K)).astype(np.int8)
+    mask = (g.random((N, K)) < 0.3).astype(np.uint8)
+    return qx, qw, mask
+
+
+def test_w8a8_integer_sum_equals_int64_matmul(oracle):
+    qx, qw, mask = _w8a8_case(3, 70, 136, 21)
+    acc, y = oracle.linear_w8a8(qx, np.ones(3, np.float32), qw, mask, np.ones(70, np.float32))
+    exact = qx.astype(np.int64) @ (qw.astype(np.int64) * mask).T
+    assert np.array_equal(acc, exact) and np.array_equal(y, exact.astype(np.float64))
+
+
+def test_w8a8_scales_by_token_and_by_row(oracle):
+    """Power-of-two scales keep everything exact: y[m, n] = acc[m, n] * 2^m * 2^-(n % 5)."""
+    M, N, K = 4, 37, 72
+    qx, qw, mask = _w8a8_case(M, N, K, 22)
+    sx = (2.0 ** np.arange(M)).astype(np.float32)
+    sw = (2.0 ** -(np.arange(N) % 5)).astype(np.float32)
+    acc, y = oracle.linear_w8a8(qx, sx, qw, mask, sw)
+    assert np.array_equal(y, acc * (2.0 ** np.arange(M))[:, None] * (2.0 ** -(np.arange(N) % 5))[None, :])
+
+
+def test_w8a8_matches_int8_weights_with_exact_bf16_activations(oracle):
+    """With sx a power of two, x = qx * sx is exact in bf16 (|qx| <= 127), and the INT8-weight
+    oracle with bf16 x must give the same float64 result (every partial sum is exact)."""
+    M, N, K = 2, 50, 200
+    qx, qw, mask = _w8a8_case(M, N, K, 23)
+    sx = np.full(M, 2.0 ** -6, np.float32)
+    sw = (np.random.default_rng(24).random(N).astype(np.float32) + 0.5) / 64
+    _, y = oracle.linear_w8a8(qx, sx, qw, mask, sw)
+    x = synth.bf16_from_f32(qx.astype(np.float32) * sx[:, None])
+    assert np.array_equal(synth.bf16_to_f32(x), qx.astype(np.float32) * sx[:, None])
+    assert np.array_equal(oracle.linear_int8(x, qw, mask, sw), y)
+
+
 # ---------------------------------------------------------------- masked update (Sec. 2.1, Algorithm 1)
 
 

@@ -27,6 +27,12 @@ MUTANTS = {
                            " + or_bf16_to_double(a[m * N + j]);"),
     "halves_row_stride": ("or_bf16_to_double(g[m * 2 * F + j]) * or_bf16_to_double(g[m * 2 * F + F + j])",
                           "or_bf16_to_double(g[m * F + j]) * or_bf16_to_double(g[m * F + F + j])"),
+    "w8a8_token_scale": ("y[m * N + n] = ((double)sx[m] * (double)sw[n]) * (double)acc;",
+                         "y[m * N + n] = ((double)sx[0] * (double)sw[n]) * (double)acc;"),
+    "w8a8_mask_dropped": ("if (mask[n * K + k]) acc += (int64_t)qx[m * K + k] * (int64_t)qw[n * K + k];",
+                          "acc += (int64_t)qx[m * K + k] * (int64_t)qw[n * K + k];"),
+    "w8a8_unsigned": ("if (mask[n * K + k]) acc += (int64_t)qx[m * K + k] * (int64_t)qw[n * K + k];",
+                      "if (mask[n * K + k]) acc += (int64_t)(uint8_t)qx[m * K + k] * (int64_t)qw[n * K + k];"),
     "update_sign": ("h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + k], w));",
                     "h = or_float_to_bf16_rne(fmaf(lr, grad[n * K + k], w));"),
     "update_truncates": ("u += 0x7FFFu + ((u >> 16) & 1u);", "u += 0u;"),
@@ -53,6 +59,8 @@ def _pin_suite(o):
         "one_hot": lambda: pins.test_linear_one_hot_selects_a_column(o),
         "int8_exact": lambda: pins.test_int8_oracle_integer_exact_and_scale(o),
         "glue": lambda: pins.test_glue_hand_derived_values(o),
+        "w8a8_int": lambda: pins.test_w8a8_integer_sum_equals_int64_matmul(o),
+        "w8a8_scales": lambda: pins.test_w8a8_scales_by_token_and_by_row(o),
         "update_rounding": lambda: pins.test_masked_update_hand_derived_rounding(o),
         "update_dense": lambda: pins.test_masked_update_equals_dense_step_then_compress(o),
     }
