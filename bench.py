@@ -54,6 +54,8 @@ def parse():
     ap.add_argument("--no-chain", action="store_true", help="skip the chained-step (glue included) section")
     ap.add_argument("--layers", type=int, default=32, help="profiling aid (--single chain): layers in the chain")
     ap.add_argument("--int8", action="store_true", help="profiling aid (--single <shape>): INT8 values + fp32 scales")
+    ap.add_argument("--update", action="store_true",
+                    help="with --single <shape>: time the masked weight update (sp_masked_update) instead of the linear")
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense cuBLAS comparison section")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
@@ -884,6 +886,9 @@ def run_single(args):
     else:
         h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
                         torch.from_numpy(mask).to(dev))
+    if args.update:
+        run_single_update(args, h, mask, dev)
+        return
     xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
     y = torch.empty((args.m, h.n), dtype=torch.bfloat16, device=dev)
     ws = torch.zeros(max(h.workspace_size(args.m), 256), dtype=torch.uint8, device=dev)
@@ -901,6 +906,45 @@ def run_single(args):
     nbytes = algorithmic_bytes(h.info, args.m, h.k, h.n)
     print(json.dumps({"single": args.single, "M": args.m, "pct": args.pct, "int8": args.int8, "us_per_launch": us,
                       "algorithmic_bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}), flush=True)
+
+
+def update_bytes(mask: np.ndarray, info) -> int:
+    """Algorithmic bytes of one masked update: the 32-byte gradient sectors (8 float32
+    columns) that hold at least one kept column, the kept values read and written, the
+    masks, and the chunk offsets."""
+    N, K = mask.shape
+    sectors = int(np.count_nonzero(mask.reshape(N, K // 8, 8).any(axis=2)))
+    return 32 * sectors + 2 * 2 * int(info.nnz) + N * K // 8 + 8 * (int(info.tiles * info.row_blocks) + 1)
+
+
+def run_single_update(args, h, mask, dev):
+    """sp_masked_update on one shape, back to back; the float32 gradient (4 bytes per
+    weight) is larger than L2 for every Llama-2-7B shape, so no flush is needed."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp
+
+    if h.dtype != "bf16":
+        raise SystemExit("--update takes bf16 weights only")
+    g = torch.randn((h.n, h.k), dtype=torch.float32, device=dev, generator=torch.Generator(dev).manual_seed(0))
+    lr = 1e-3
+    for _ in range(args.warmup):
+        h.masked_update(g, lr)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        h.masked_update(g, lr)
+    b.record()
+    torch.cuda.synchronize()
+    sp.check()
+    us = a.elapsed_time(b) / max(args.steps, 1) * 1e3
+    nbytes = update_bytes(mask, h.info)
+    peak, kind = load_peaks()
+    gbs = nbytes / (us * 1e-6) / 1e9
+    print(json.dumps({"single": args.single, "op": "masked_update", "pct": args.pct, "us_per_launch": us,
+                      "algorithmic_bytes": nbytes, "gbs": gbs, "frac": gbs / peak, "peak_gbs": peak,
+                      "peak_kind": kind}), flush=True)
 
 
 def main():

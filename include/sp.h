@@ -163,6 +163,20 @@ sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* 
  *   wrong results; order them on one stream. */
 sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* stream);
 
+/* The masked weight step of sparse training (Sec. 2.1, Algorithm 1) applied in place to
+ * the compressed form: every kept weight becomes
+ *     w[n,k] <- bf16_rne(fma(-lr, grad[n,k], w[n,k]))      (float32, one rounding)
+ * and masked-out weights stay zero, since the mask never changes.  Only the packed values
+ * are rewritten; masks, chunk offsets, padding and the handle's metadata stay as they are,
+ * so the handle stays valid for every other call.
+ *   grad_dev   [N, K] float32, dense and row-major; its masked-out entries are not read
+ *              (a 32-byte sector all of whose columns are masked out is not fetched).
+ *   lr         the step size (any finite float; 0 leaves the values unchanged).
+ * bf16 handles only (SP_ERR_UNSUPPORTED for SP_INT8).  Asynchronous on `stream`; work
+ * that reads the handle (sp_linear, sp_decompress, ...) must be ordered after it by the
+ * caller.  No allocation, no host sync.  Results are bitwise deterministic. */
+sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float lr, void* stream);
+
 /* A copy of the handle with its own device buffers (same bytes), allocated on the
  * current device, which must be the handle's (SP_ERR_INVALID_ARG otherwise).  The copies
  * run on `stream`, which is synchronised before the call returns. */

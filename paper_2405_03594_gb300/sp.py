@@ -25,7 +25,7 @@ STATUS = {
 }
 # every function declared in include/sp.h and include/sp_stack.h
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
-           "sp_linear_noalloc",
+           "sp_linear_noalloc", "sp_masked_update",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
            "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_chain_workspace_size", "sp_chain_run"]
 
@@ -70,6 +70,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_linear.argtypes = [P, P, I64, P, P, SZ, P]
     lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
     lib.sp_linear_noalloc.argtypes = [P, P, I64, P, P]
+    lib.sp_masked_update.argtypes = [P, P, ctypes.c_float, P]
     lib.sp_clone.argtypes = [P, ALLOC_FN, FREE_FN, P, P, ctypes.POINTER(P)]
     lib.sp_free.argtypes = [P]
     lib.sp_info.argtypes = [P, ctypes.POINTER(SpInfo)]
@@ -186,6 +187,14 @@ class SparseMatrix:
         assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
         _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)), "sp_linear_noalloc")
         return out
+
+    def masked_update(self, grad: torch.Tensor, lr: float, stream=None) -> "SparseMatrix":
+        """sp_masked_update: w <- bf16(fma(-lr, grad, w)) on every kept weight, in place on
+        the compressed values (Algorithm 1's masked step); grad [N, K] float32 on this
+        matrix's device."""
+        assert grad.dtype == torch.float32 and grad.shape == (self.n, self.k) and grad.is_contiguous()
+        _check(_lib.sp_masked_update(self._h, _ptr(grad), float(lr), _stream(stream)), "sp_masked_update")
+        return self
 
     def decompress(self, stream=None) -> torch.Tensor:
         dt = torch.int8 if self.dtype == "int8" else torch.bfloat16
