@@ -58,6 +58,7 @@ def parse():
                     help="with --single <shape>: time the masked weight update (sp_masked_update) instead of the linear")
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense cuBLAS comparison section")
+    ap.add_argument("--no-update", action="store_true", help="skip the masked weight update section")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
                     help="profiling aid: time one layer-0 linear of this shape, or the chained step of --layers "
                          "layers (--warmup then --steps launches)")
@@ -820,6 +821,7 @@ def run_ours(args):
     stack = None if (args.no_stack or world > 1) else stack_section(args, peak_gbs, host_bf)
     prefill = None if (args.no_prefill or world > 1) else prefill_section(args)
     dense = None if (args.no_dense or world > 1) else dense_section(host, xs, results, Ms)
+    update = None if (args.no_update or world > 1) else update_section(args, host, peak_gbs)
 
     if rank == 0:
         launches_per_step = LAYERS * sum(launch_counts.values())
@@ -849,6 +851,7 @@ def run_ours(args):
             "stack_int8": stack,
             "prefill": prefill,
             "dense_comparison": dense,
+            "masked_update": update,
             "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
                                "frac_of_peak": v["step_gbs"] / peak_gbs,
                                "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),
@@ -915,6 +918,46 @@ def update_bytes(mask: np.ndarray, info) -> int:
     N, K = mask.shape
     sectors = int(np.count_nonzero(mask.reshape(N, K // 8, 8).any(axis=2)))
     return 32 * sectors + 2 * 2 * int(info.nnz) + N * K // 8 + 8 * (int(info.tiles * info.row_blocks) + 1)
+
+
+def update_section(args, host, peak_gbs):
+    """Masked weight update (Algorithm 1's step on the compressed form) on the layer-0
+    weights of the four shapes: back-to-back sp_masked_update launches; the float32
+    gradients (4 bytes per weight) are larger than L2.  Context next to the decode step;
+    a failure here is reported in the section and never ends the run."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp
+
+    dev = torch.device("cuda", 0)
+    res = {"kernel": "masked_update_kernel", "lr": 1e-3, "peak_gbs": peak_gbs, "shapes": {}}
+    try:
+        for name in SHAPES:
+            W, mask, _ = host[name]
+            h = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
+                            torch.from_numpy(mask).to(dev))
+            g = torch.randn((h.n, h.k), dtype=torch.float32, device=dev,
+                            generator=torch.Generator(dev).manual_seed(0))
+            for _ in range(3):
+                h.masked_update(g, 1e-3)
+            torch.cuda.synchronize()
+            reps = 20
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(reps):
+                h.masked_update(g, 1e-3)
+            b.record()
+            torch.cuda.synchronize()
+            sp.check()
+            us = a.elapsed_time(b) / reps * 1e3
+            nbytes = update_bytes(mask, h.info)
+            gbs = nbytes / (us * 1e-6) / 1e9
+            res["shapes"][name] = {"us": us, "algorithmic_bytes": nbytes, "gbs": gbs, "frac": gbs / peak_gbs}
+            del h, g
+        torch.cuda.empty_cache()
+    except Exception as e:  # context only: never let it end the run
+        res["error"] = f"{type(e).__name__}: {e}"
+    return res
 
 
 def run_single_update(args, h, mask, dev):

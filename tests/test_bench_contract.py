@@ -127,3 +127,28 @@ def test_dense_section_reports_failures_instead_of_raising():
     out = b.dense_section({}, {}, {}, [1])
     assert "error" in out and out["paper"]["gpu_sparsity_only"]["x"] == 1.7
     assert out["shapes"] == {} and out["step_speedup"] == {}
+
+
+def test_update_bytes_counts_gradient_sectors_values_masks_and_offsets():
+    """Roofline bytes of one masked update, by hand: a 128 x 64 matrix (one chunk) whose
+    row 0 keeps columns 0 and 9 and row 1 keeps column 63: gradient sectors of 8 columns
+    holding a kept column are (0, 0), (0, 1) and (1, 7), so 3 x 32 bytes; 3 kept values are
+    read and written (3 x 4 bytes); the masks are 128 x 64 / 8 bytes; 2 chunk offsets."""
+    import numpy as np
+
+    b = _bench_module()
+    mask = np.zeros((128, 64), dtype=np.uint8)
+    mask[0, 0] = mask[0, 9] = mask[1, 63] = 1
+
+    class Info:
+        nnz, tiles, row_blocks = 3, 1, 1
+
+    assert b.update_bytes(mask, Info) == 3 * 32 + 3 * 4 + 128 * 64 // 8 + 2 * 8
+
+
+def test_update_section_reports_failures_instead_of_raising():
+    """The masked-update section is context next to the decode step: without a GPU it
+    returns its failure inside the section rather than ending the run."""
+    b = _bench_module()
+    out = b.update_section(None, {n: (None, None, None) for n in b.SHAPES}, 6681.8)
+    assert "error" in out and out["shapes"] == {} and out["kernel"] == "masked_update_kernel"
