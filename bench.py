@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense cuBLAS comparison section")
     ap.add_argument("--no-update", action="store_true", help="skip the masked weight update section")
+    ap.add_argument("--no-sweep-config", action="store_true",
+                    help="skip the sparsity x batch sweep (gate_up/down, non-uniform masks, M = 1..256)")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
                     help="profiling aid: time one layer-0 linear of this shape, or the chained step of --layers "
                          "layers (--warmup then --steps launches)")
@@ -770,6 +772,7 @@ def run_ours(args):
     prefill = None if (args.no_prefill or world > 1) else prefill_section(args)
     dense = None if (args.no_dense or world > 1) else dense_section(host, xs, results, Ms)
     update = None if (args.no_update or world > 1) else update_section(args, host, peak_gbs)
+    sweep = None if (args.no_sweep_config or world > 1) else sweep_section(args, peak_gbs)
 
     if rank == 0:
         launches_per_step = LAYERS * sum(launch_counts.values())
@@ -800,6 +803,7 @@ def run_ours(args):
             "prefill": prefill,
             "dense_comparison": dense,
             "masked_update": update,
+            "sparsity_batch_sweep": sweep,
             "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
                                "frac_of_peak": v["step_gbs"] / peak_gbs,
                                "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),
@@ -866,6 +870,84 @@ def update_bytes(mask: np.ndarray, info) -> int:
     N, K = mask.shape
     sectors = int(np.count_nonzero(mask.reshape(N, K // 8, 8).any(axis=2)))
     return 32 * sectors + 2 * 2 * int(info.nnz) + N * K // 8 + 8 * (int(info.tiles * info.row_blocks) + 1)
+
+
+SWEEP_SHAPES = ("gate_up", "down")
+SWEEP_PCTS = (0, 50, 60, 70, 80)
+SWEEP_MS = (1, 2, 4, 8, 16, 32, 64, 128, 256)
+
+
+def sweep_copies(compressed_bytes: int) -> int:
+    """Distinct device copies of one matrix so that a graph of launches over them reads
+    more than 3x L2 of compressed weights (no L2 flush needed between launches)."""
+    return max(2, -(-int(3 * L2_BYTES) // max(int(compressed_bytes), 1)))
+
+
+def roofline_time_us(nbytes: int, nnz: int, M: int, hbm_gbs: float, tensor_tflops: float) -> tuple[float, str]:
+    """The slower of the compressed bytes over the HBM peak and the nonzero FLOPs
+    (2 M nnz) over the bf16 tensor peak, in microseconds, and which one it is."""
+    t_bytes = nbytes / (hbm_gbs * 1e9) * 1e6
+    t_flops = 2.0 * M * nnz / (tensor_tflops * 1e12) * 1e6
+    return (t_bytes, "hbm") if t_bytes >= t_flops else (t_flops, "tensor")
+
+
+def sweep_section(args, peak_gbs):
+    """The sparsity x batch sweep: gate_up 4096->22016 and down 11008->4096, non-uniform
+    masks (per-row sparsity within +-10 points of the target, 5% dense input columns) at
+    0/50/60/70/80%, M = 1 ... 256 on the automatic kernel choice.  Each point is a CUDA graph
+    of launches over enough distinct copies to read > 3x L2; per-launch time, GB/s, and the
+    fraction of the roofline (the slower of bytes over HBM peak and nonzero FLOPs over the
+    bf16 tensor peak).  Parity of the same inputs is checked by the GPU tests."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+
+    tensor_peak, tkind = load_tensor_peak()
+    dev = torch.device("cuda", 0)
+    res = {"workload": "gate_up 4096->22016 and down 11008->4096, non-uniform per-row magnitude masks "
+                       "(+-10 points, 5% dense columns), bf16, auto kernel",
+           "hbm_peak_gbs": peak_gbs, "tensor_peak_tflops": tensor_peak, "tensor_peak_kind": tkind, "points": {}}
+    try:
+        for name in SWEEP_SHAPES:
+            N, K = synth.LLAMA2_7B_SHAPES[name]
+            p = synth.PROJ_IDS[name]
+            W = synth.weight(N, K, synth.rng(0, 0, p, synth.STREAM_W))
+            x = synth.activations(max(SWEEP_MS), K, synth.rng(0, 0, p, synth.STREAM_X))
+            xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+            for pct in SWEEP_PCTS:
+                mask, _, _ = synth.nonuniform_mask(W, pct, synth.rng(0, 0, p, synth.STREAM_MASK))
+                h0 = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
+                                 torch.from_numpy(mask).to(dev))
+                copies = sweep_copies(int(h0.info.bytes))
+                hs = [h0] + [h0.clone() for _ in range(copies - 1)]
+                y = torch.empty((max(SWEEP_MS), N), dtype=torch.bfloat16, device=dev)
+                ws = torch.zeros(max(max(h0.workspace_size(M) for M in SWEEP_MS), 256), dtype=torch.uint8, device=dev)
+                pts = {}
+                for M in SWEEP_MS:
+                    for h in hs:
+                        h.linear(xd[:M], out=y[:M], workspace=ws)
+                    torch.cuda.synchronize()
+                    g = torch.cuda.CUDAGraph()
+                    with torch.cuda.graph(g):
+                        for h in hs:
+                            h.linear(xd[:M], out=y[:M], workspace=ws)
+                    ms = time_graph(g, 10, 3)
+                    sp.check()
+                    us = ms * 1e3 / copies
+                    nbytes = algorithmic_bytes(h0.info, M, K, N)
+                    t_roof, bound = roofline_time_us(nbytes, int(h0.info.nnz), M, peak_gbs, tensor_peak)
+                    pts[str(M)] = {"us": us, "tok_s": M / (us * 1e-6), "gbs": nbytes / (us * 1e-6) / 1e9,
+                                   "tflops_nonzero": 2.0 * M * int(h0.info.nnz) / (us * 1e-6) / 1e12,
+                                   "bound": bound, "frac_of_roofline": t_roof / us,
+                                   "kernel": h0.kernel_name(M)}
+                    del g
+                res["points"][f"{name}@{pct}%"] = {"copies": copies, "nnz": int(h0.info.nnz),
+                                                   "compressed_bytes": int(h0.info.bytes), "by_m": pts}
+                del hs, h0, y, ws
+                torch.cuda.empty_cache()
+    except Exception as e:  # context only: never let it end the run
+        res["error"] = f"{type(e).__name__}: {e}"
+    return res
 
 
 def update_section(args, host, peak_gbs):

@@ -152,3 +152,29 @@ def test_update_section_reports_failures_instead_of_raising():
     b = _bench_module()
     out = b.update_section(None, {n: (None, None, None) for n in b.SHAPES}, 6681.8)
     assert "error" in out and out["shapes"] == {} and out["kernel"] == "masked_update_kernel"
+
+
+def test_sweep_copies_exceed_three_l2():
+    """A graph over the sweep's copies reads more than 3x L2 of distinct compressed bytes."""
+    b = _bench_module()
+    for nbytes in (10_000_000, 45_000_000, 65_400_000, 191_600_000, 500_000_000):
+        c = b.sweep_copies(nbytes)
+        assert c * nbytes > 3 * b.L2_BYTES  # enough copies
+        assert c == 2 or (c - 1) * nbytes <= 3 * b.L2_BYTES  # and no more than needed (at least 2)
+
+
+def test_roofline_time_takes_the_slower_bound():
+    """Bytes over HBM peak against nonzero FLOPs over tensor peak, by hand: 66.2 MB at
+    6681.8 GB/s is 9.907 us; 2 * 256 * 27e6 FLOPs at 1936.4 TFLOP/s is 7.14 us (HBM-bound),
+    and at M = 2048 the FLOPs (57.1 us) win."""
+    b = _bench_module()
+    t, bound = b.roofline_time_us(66_200_000, 27_000_000, 256, 6681.8, 1936.4)
+    assert bound == "hbm" and t == pytest.approx(66.2e6 / 6681.8e9 * 1e6)
+    t, bound = b.roofline_time_us(66_200_000, 27_000_000, 2048, 6681.8, 1936.4)
+    assert bound == "tensor" and t == pytest.approx(2 * 2048 * 27e6 / 1936.4e12 * 1e6)
+
+
+def test_sweep_section_reports_failures_instead_of_raising():
+    b = _bench_module()
+    out = b.sweep_section(None, 6681.8)
+    assert "error" in out and out["points"] == {}
