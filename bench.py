@@ -59,6 +59,8 @@ def parse():
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense cuBLAS comparison section")
     ap.add_argument("--no-update", action="store_true", help="skip the masked weight update section")
+    ap.add_argument("--square-sweep", action="store_true",
+                    help="run only the 12288 x 12288 sparse matmul at 0-90%% sparsity (M = 2048, tensor cores)")
     ap.add_argument("--no-sweep-config", action="store_true",
                     help="skip the sparsity x batch sweep (gate_up/down, non-uniform masks, M = 1..256)")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
@@ -863,6 +865,57 @@ def run_single(args):
                       "algorithmic_bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}), flush=True)
 
 
+def run_square_sweep(args):
+    """The 12288 x 12288 sparse matmul against sparsity (the scaling example of Sec. 2.3 and its
+    12K x 12K figure, measured there on a CS-3; run here on the tensor-core kernel): x [2048, 12288] bf16, per-row magnitude masks at
+    0, 10, ..., 90 %, y = x . (W o M)^T.  Prints one JSON line: per sparsity the launch time,
+    its speedup over the 0 % matrix through the same kernel, the ideal 1 / (1 - s), and the
+    dense cuBLAS GEMM of the same shape for reference.  Opt-in (--square-sweep)."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+
+    dev = torch.device("cuda", 0)
+    N = K = 12288
+    M = 2048
+    W = synth.weight(N, K, synth.rng(0, 0, 0, synth.STREAM_W))
+    x = synth.activations(M, K, synth.rng(0, 0, 0, synth.STREAM_X))
+    xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    reps = max(3, min(args.steps, 20))
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(reps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps * 1e3
+
+    Wd = torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16)
+    dense_us = timed(lambda: torch.matmul(xd, Wd.t()))
+    out = {"single": "square_sweep", "N": N, "K": K, "M": M, "kernel": "linear_tc_kernel",
+           "dense_cublas_us": dense_us, "points": {}}
+    base = None
+    for pct in range(0, 100, 10):
+        mask = synth.magnitude_mask(W, pct)
+        h = sp.compress(Wd, torch.from_numpy(mask).to(dev))
+        ws = torch.zeros(max(h.workspace_size(M), 256), dtype=torch.uint8, device=dev)
+        us = timed(lambda: h.linear(xd, out=y, workspace=ws, path="tensor_core"))
+        sp.check()
+        base = us if base is None else base
+        out["points"][str(pct)] = {"us": us, "speedup_vs_0pct": base / us, "ideal": 1.0 / (1.0 - pct / 100.0),
+                                   "speedup_vs_dense_cublas": dense_us / us, "nnz": int(h.info.nnz),
+                                   "compressed_bytes": int(h.info.bytes)}
+        del h, ws
+        torch.cuda.empty_cache()
+    print(json.dumps(out), flush=True)
+
+
 def update_bytes(mask: np.ndarray, info) -> int:
     """Algorithmic bytes of one masked update: the 32-byte gradient sectors (8 float32
     columns) that hold at least one kept column, the kept values read and written, the
@@ -1022,6 +1075,9 @@ def run_single_update(args, h, mask, dev):
 
 def main():
     args = parse()
+    if args.square_sweep:
+        run_square_sweep(args)
+        return
     if args.single:
         run_single(args)
         return
