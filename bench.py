@@ -967,10 +967,10 @@ def sweep_section(args, peak_gbs):
             W = synth.weight(N, K, synth.rng(0, 0, p, synth.STREAM_W))
             x = synth.activations(max(SWEEP_MS), K, synth.rng(0, 0, p, synth.STREAM_X))
             xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+            Wd = torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16)
             for pct in SWEEP_PCTS:
                 mask, _, _ = synth.nonuniform_mask(W, pct, synth.rng(0, 0, p, synth.STREAM_MASK))
-                h0 = sp.compress(torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16),
-                                 torch.from_numpy(mask).to(dev))
+                h0 = sp.compress(Wd, torch.from_numpy(mask).to(dev))
                 copies = sweep_copies(int(h0.info.bytes))
                 hs = [h0] + [h0.clone() for _ in range(copies - 1)]
                 y = torch.empty((max(SWEEP_MS), N), dtype=torch.bfloat16, device=dev)
@@ -998,8 +998,10 @@ def sweep_section(args, peak_gbs):
                                                    "compressed_bytes": int(h0.info.bytes), "by_m": pts}
                 del hs, h0, y, ws
                 torch.cuda.empty_cache()
+            del Wd, xd
     except Exception as e:  # context only: never let it end the run
         res["error"] = f"{type(e).__name__}: {e}"
+    torch.cuda.empty_cache()
     return res
 
 
