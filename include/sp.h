@@ -177,6 +177,28 @@ sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, vo
  * caller.  No allocation, no host sync.  Results are bitwise deterministic. */
 sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float lr, void* stream);
 
+/* INT8 weights and INT8 activations (Sec. 3.4, the sparse INT8 deployment):
+ *     y[m,n] = bf16_rne(sx[m] * sw[n] * sum_k qx[m,k] * qw[n,k] * Mask[n,k])
+ * for a handle compressed from SP_INT8 values qw with per-row scales sw.  On GB300 the dense
+ * INT8 tensor rate is far below the bf16 rate, so the activations are widened once,
+ * x[m,k] = bf16_rne(qx[m,k] * sx[m]) (float32 product), into the workspace, and the
+ * INT8-weight sparse linear of sp_linear runs on that x: FP32 accumulation, sw applied in
+ * its epilogue, one bf16 rounding of y.
+ *   qx_dev     [m, K] int8, row-major.        sx_dev [m] fp32 per-token scales.
+ *   y_dev      [m, N] bf16 (fully overwritten).
+ *   workspace  at least sp_w8a8_workspace_size(h, m) bytes, zero-filled before its first
+ *              use: sp_linear's workspace for (h, m) followed by the widened activations,
+ *              so one buffer can serve sp_linear and sp_linear_w8a8 calls ordered on one
+ *              stream.
+ * SP_ERR_UNSUPPORTED for a bf16 handle; otherwise the errors of sp_linear.  m == 0 returns
+ * SP_OK without a launch.  Two launches (widening, linear), no allocation, no host sync. */
+sp_status sp_linear_w8a8(const sp_matrix* h, const int8_t* qx_dev, const float* sx_dev, int64_t m, void* y_dev,
+                         void* workspace_dev, size_t workspace_bytes, void* stream);
+
+/* Workspace bytes sp_linear_w8a8 needs for a batch of m rows (0 for m == 0).  Host only.
+ * SP_ERR_INVALID_ARG for m < 0 or a null `bytes`, SP_ERR_BAD_HANDLE for a dead handle. */
+sp_status sp_w8a8_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
+
 /* A copy of the handle with its own device buffers (same bytes), allocated on the
  * current device, which must be the handle's (SP_ERR_INVALID_ARG otherwise).  The copies
  * run on `stream`, which is synchronised before the call returns. */

@@ -25,7 +25,7 @@ STATUS = {
 }
 # every function declared in include/sp.h and include/sp_stack.h
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
-           "sp_linear_noalloc", "sp_masked_update",
+           "sp_linear_noalloc", "sp_masked_update", "sp_linear_w8a8", "sp_w8a8_workspace_size",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
            "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_chain_workspace_size", "sp_chain_run"]
 
@@ -71,6 +71,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
     lib.sp_linear_noalloc.argtypes = [P, P, I64, P, P]
     lib.sp_masked_update.argtypes = [P, P, ctypes.c_float, P]
+    lib.sp_linear_w8a8.argtypes = [P, P, P, I64, P, P, SZ, P]
+    lib.sp_w8a8_workspace_size.argtypes = [P, I64, ctypes.POINTER(SZ)]
     lib.sp_clone.argtypes = [P, ALLOC_FN, FREE_FN, P, P, ctypes.POINTER(P)]
     lib.sp_free.argtypes = [P]
     lib.sp_info.argtypes = [P, ctypes.POINTER(SpInfo)]
@@ -186,6 +188,26 @@ class SparseMatrix:
         assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
         assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
         _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)), "sp_linear_noalloc")
+        return out
+
+    def w8a8_workspace_size(self, m: int) -> int:
+        b = ctypes.c_size_t()
+        _check(_lib.sp_w8a8_workspace_size(self._h, m, ctypes.byref(b)), "sp_w8a8_workspace_size")
+        return int(b.value)
+
+    def linear_w8a8(self, qx: torch.Tensor, sx: torch.Tensor, out: torch.Tensor | None = None,
+                    workspace: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """sp_linear_w8a8: y = sx[m] * sw[n] * (qx . (qw o Mask)^T) for an INT8 matrix, with
+        qx [m, K] int8 and sx [m] fp32 per-token scales on this matrix's device."""
+        assert qx.dtype == torch.int8 and qx.dim() == 2 and qx.shape[1] == self.k and qx.is_contiguous()
+        assert sx.dtype == torch.float32 and sx.shape == (qx.shape[0],) and sx.is_contiguous()
+        m = qx.shape[0]
+        if out is None:
+            out = torch.empty((m, self.n), dtype=torch.bfloat16, device=qx.device)
+        if workspace is None:
+            workspace = workspace_for(self.w8a8_workspace_size(m), qx.device)
+        _check(_lib.sp_linear_w8a8(self._h, _ptr(qx), _ptr(sx), m, _ptr(out), _ptr(workspace), workspace.numel(),
+                                   _stream(stream)), "sp_linear_w8a8")
         return out
 
     def masked_update(self, grad: torch.Tensor, lr: float, stream=None) -> "SparseMatrix":

@@ -158,6 +158,16 @@ def quantize_int8(W: np.ndarray, mask: np.ndarray):
     return q, s
 
 
+def quantize_activations_int8(x: np.ndarray):
+    """(qx int8 [M, K], sx float32 [M]) by symmetric absmax per token (row of x, bf16 bits):
+    sx = max|x_m| / 127 (1 for an all-zero row), qx = clamp(rne(x / sx), -127, 127)."""
+    xf = bf16_to_f32(x).astype(np.float64)
+    amax = np.abs(xf).max(axis=1)
+    sx = np.where(amax > 0, amax / 127.0, 1.0).astype(np.float32)
+    qx = np.clip(np.rint(xf / sx.astype(np.float64)[:, None]), -127, 127).astype(np.int8)
+    return qx, sx
+
+
 def layer_inputs(shape_name: str, pct: int, M: int, seed: int = 0, layer: int = 0):
     """(W, mask, x) for one Llama-2-7B linear at a uniform per-row sparsity."""
     N, K = LLAMA2_7B_SHAPES[shape_name]

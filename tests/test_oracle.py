@@ -430,3 +430,21 @@ def test_quantize_int8_properties():
     assert s[3] == 1.0 and not q[3].any()
     assert (np.abs(q).max(axis=1)[np.arange(50) != 3] == 127).all()
     assert not q[mask == 0].any()
+
+
+def test_per_token_activation_quantization_recipe():
+    """The harness's INT8 activations (symmetric absmax per token): the largest |x| of a row
+    maps to +-127 exactly, every code is within [-127, 127], and dequantizing is within half
+    a step of x; an all-zero row gets scale 1 and zero codes."""
+    from paper_2405_03594_gb300 import synth
+
+    x = synth.activations(6, 200, np.random.default_rng(0))
+    x[5] = 0
+    qx, sx = synth.quantize_activations_int8(x)
+    xf = synth.bf16_to_f32(x).astype(np.float64)
+    assert qx.dtype == np.int8 and sx.dtype == np.float32 and np.abs(qx.astype(int)).max() <= 127
+    for m in range(5):
+        j = np.abs(xf[m]).argmax()
+        assert abs(int(qx[m, j])) == 127
+        assert np.abs(qx[m] * np.float64(sx[m]) - xf[m]).max() <= 0.5 * sx[m] * (1 + 1e-6)
+    assert sx[5] == 1 and not qx[5].any()
