@@ -325,8 +325,8 @@ def dense_section(host, xs, results, Ms):
 
 
 # The source files that compile into each profiled kernel (its translation unit and the
-# device headers it includes, plus the public headers without their comments); host-only
-# files such as sp_api.cu do not change the kernel.
+# device headers it includes, plus the public headers without their comments and function
+# prototypes); host-only files such as sp_api.cu do not change the kernel.
 KERNEL_SOURCES = {
     "linear_ccw_kernel": ("sp_linear_cc.cu", "sp_cc_common.cuh", "sp_internal.cuh"),
     "linear_cc_kernel": ("sp_linear_cc.cu", "sp_cc_common.cuh", "sp_internal.cuh"),
@@ -348,6 +348,8 @@ def kernel_source_hash(kernel: str):
     for n in ("sp.h", "sp_stack.h"):
         with open(os.path.join(ROOT, "include", n)) as f:
             code = re.sub(r"/\*.*?\*/|//[^\n]*", "", f.read(), flags=re.S)
+        # function prototypes declare host entry points and compile into no kernel
+        code = re.sub(r"(?:sp_status|const\s+char\s*\*)\s*sp_\w+\s*\([^;{}]*\)\s*;", "", code)
         h.update(n.encode() + b"\0" + " ".join(code.split()).encode())
     return h.hexdigest()[:16]
 

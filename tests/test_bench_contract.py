@@ -53,8 +53,9 @@ def _bench_module():
 
 
 def test_traffic_staleness_hash_follows_the_kernel_sources(tmp_path):
-    """The committed ncu traffic stays valid across host-only edits and comment edits of
-    the public headers, and is dropped once a source of the kernel itself changes."""
+    """The committed ncu traffic stays valid across host-only edits, comment edits and new
+    function prototypes in the public headers, and is dropped once a source of the kernel
+    itself, or a type or constant of the headers, changes."""
     import shutil
 
     b = _bench_module()
@@ -72,6 +73,8 @@ def test_traffic_staleness_hash_follows_the_kernel_sources(tmp_path):
 
     edit("paper_2405_03594_gb300/csrc/sp_api.cu", "extern \"C\" {", "extern \"C\" {\n// host-only edit")
     edit("include/sp.h", "/*", "/* comment edit;")
+    edit("include/sp.h", "#ifdef __cplusplus\n}", "sp_status sp_new_entry(const sp_matrix* h,\n  int64_t m);\n"
+         "#ifdef __cplusplus\n}")
     assert {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES} == base
     edit("paper_2405_03594_gb300/csrc/sp_linear_tc.cu", "namespace sp {", "namespace sp {\nstatic int edited;")
     now = {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES}
@@ -79,6 +82,9 @@ def test_traffic_staleness_hash_follows_the_kernel_sources(tmp_path):
     assert all(now[k] == base[k] for k in base if k != "linear_tc_kernel")
     edit("include/sp.h", "#define", "#define SP_EDITED 1\n#define")
     assert all(b.kernel_source_hash(k) != base[k] for k in base)
+    mid = {k: b.kernel_source_hash(k) for k in b.KERNEL_SOURCES}
+    edit("include/sp.h", "SP_ERR_WORKSPACE = 8", "SP_ERR_WORKSPACE = 9")
+    assert all(b.kernel_source_hash(k) != mid[k] for k in base)
 
 
 def test_committed_traffic_matches_the_current_kernel_sources():
