@@ -188,6 +188,25 @@ def test_config_llama_shapes_70pct_decode(sp, oracle, name):
     sp.check()
 
 
+@pytest.mark.parametrize("name", list(synth.LLAMA2_7B_SHAPES))
+@pytest.mark.parametrize("pct", [50, 70])
+def test_config_prefill_2048_sampled(sp, oracle, name, pct):
+    """Prefill: the four shapes at 50% and 70%, x [2048, K], on the tensor-core kernel with
+    the inputs and launch the bench's prefill section times; the oracle computes 64 output
+    rows (all 2048 tokens each), the first and last included."""
+    W, mask, _ = synth.layer_inputs(name, pct, 1, seed=0, layer=0)
+    N, K = W.shape
+    x = synth.activations(2048, K, synth.rng(0, 0, synth.PROJ_IDS[name], synth.STREAM_X))
+    _, y = _run(sp, W, None, mask, x, path="tensor_core")
+    rows = np.sort(np.random.default_rng(pct + N).choice(N, 64, replace=False))
+    rows[0], rows[-1] = 0, N - 1
+    ref = oracle.linear_bf16(x, W[rows], mask[rows])
+    import torch
+
+    got = gu.bf16_from_dev(y[:, torch.from_numpy(rows).to(y.device)])
+    gu.assert_close(got, ref, f"prefill {name} {pct}% M=2048")
+
+
 @pytest.mark.parametrize("name", ["gate_up", "down"])
 @pytest.mark.parametrize("pct", [0, 50, 60, 70, 80])
 def test_config_sweep_nonuniform_sampled(sp, oracle, name, pct):
