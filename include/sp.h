@@ -171,7 +171,8 @@ sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, vo
  * so the handle stays valid for every other call.
  *   grad_dev   [N, K] float32, dense and row-major; the values of its masked-out
  *              entries are never used (they may hold anything, NaN included).
- *   lr         the step size (any finite float; 0 leaves the values unchanged).
+ *   lr         the step size, finite (SP_ERR_INVALID_ARG otherwise); 0 leaves the values
+ *              unchanged.
  * bf16 handles only (SP_ERR_UNSUPPORTED for SP_INT8).  Asynchronous on `stream`; work
  * that reads the handle (sp_linear, sp_decompress, ...) must be ordered after it by the
  * caller.  No allocation, no host sync.  Results are bitwise deterministic. */

@@ -118,7 +118,7 @@ using namespace sp;
 
 extern "C" sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float lr, void* stream) {
   if (!h || h->magic != SP_MAGIC) return SP_ERR_BAD_HANDLE;
-  if (!grad_dev) return SP_ERR_INVALID_ARG;
+  if (!grad_dev || !isfinite(lr)) return SP_ERR_INVALID_ARG;
   if (h->dtype != SP_BF16) return SP_ERR_UNSUPPORTED;
   if (!aligned16(grad_dev)) return SP_ERR_ALIGNMENT;
   int dev = -1;

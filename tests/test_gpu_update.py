@@ -126,6 +126,8 @@ def test_argument_errors(sp):
     import ctypes
 
     assert lib.sp_masked_update(h.handle, None, ctypes.c_float(0.1), None) == 1  # null gradient
+    assert lib.sp_masked_update(h.handle, ctypes.c_void_p(gd.data_ptr()), ctypes.c_float(float("nan")), None) == 1
+    assert lib.sp_masked_update(h.handle, ctypes.c_void_p(gd.data_ptr()), ctypes.c_float(float("inf")), None) == 1
     assert lib.sp_masked_update(h.handle, ctypes.c_void_p(gd.data_ptr() + 4), ctypes.c_float(0.1), None) == 3
     q, s = synth.quantize_int8(W, mask)
     hi = sp.compress(gu.i8_to_dev(q), gu.u8_to_dev(mask), gu.f32_to_dev(s))
