@@ -14,7 +14,9 @@ prefill.
   python bench.py [--gpus N --steps K --warmup W --m M]        our CUDA path
   python bench.py --impl reference ...                          the float64 CPU oracle
 
-One JSON line on stdout (rank 0).  With --gpus N > 1 (under torchrun) every rank
+One compact JSON line on stdout (rank 0, about 2 KB: the headline figures, the roofline of
+the dominant kernel, the CPU baseline, clocks and a summary of the context sections; the
+sections in full go to --sections-out).  With --gpus N > 1 (under torchrun) every rank
 runs an independent replica (weak scaling; no collective on the data path).
 """
 from __future__ import annotations
@@ -63,6 +65,9 @@ def parse():
                     help="run only the 12288 x 12288 sparse matmul at 0-90%% sparsity (M = 2048, tensor cores)")
     ap.add_argument("--no-sweep-config", action="store_true",
                     help="skip the sparsity x batch sweep (gate_up/down, non-uniform masks, M = 1..256)")
+    ap.add_argument("--sections-out", default="",
+                    help="write the full context sections (per-M tables, chained step, INT8 stack, prefill, dense "
+                         "comparison, masked update, sweep) to this JSON file; the stdout line carries a summary")
     ap.add_argument("--single", default="", choices=["", "chain", *SHAPES],
                     help="profiling aid: time one layer-0 linear of this shape, or the chained step of --layers "
                          "layers (--warmup then --steps launches)")
@@ -441,57 +446,52 @@ def cpu_oracle_leg(host, M: int, reps_target_s: float = 10.0):
             break
     t = sorted(t_layer)[len(t_layer) // 2]
     return ({"value": M / (LAYERS * t), "unit": "tok/s", "cores": cores, "kind": "oracle",
-             "sample": f"layer 0 of {LAYERS} (qkv, o, gate_up, down) at M={M}, float64 C oracle with OpenMP over "
-                       f"output rows, median of {len(t_layer)} runs of {t:.2f} s, scaled x{LAYERS} to one step"},
+             "sample": f"layer 0 (qkv, o, gate_up, down) at M={M}, float64 C oracle, OpenMP over rows; "
+                       f"median of {len(t_layer)} runs of {t:.2f} s, x{LAYERS} layers"},
             outs)
 
 
-REF_ROW_FRACTION = 8  # each reference step computes 1/8 of every layer-0 output row set
-
-
 def run_reference(args):
-    """The float64 oracle on the host cores, on the same workload: each step computes
-    every 8th output row of the four layer-0 linears (a bounded sample), and the time is
-    scaled by 8 x 32 to a full 32-layer step."""
+    """The float64 oracle on the host cores, on the same workload as our arm: one step is
+    the full decode step, the four layer-0 linears (qkv, o, gate_up, down) computed for
+    each of the 32 layers at M rows -- the same 128 products and the same bytes that our
+    arm's step streams (its 32 layers are copies of layer 0 too).  Nothing is sampled or
+    extrapolated: the timed region is exactly `steps` such steps."""
     rank, _, world = dist_env()
     if rank != 0:
         return
     host = host_layer(args.pct, args.m)
     cores = len(os.sched_getaffinity(0))
     os.environ.setdefault("OMP_NUM_THREADS", str(cores))
-    import numpy as np
-
     import oracle
 
-    sample = {}
-    for name in SHAPES:
-        W, mask, x = host[name]
-        rows = np.arange(0, W.shape[0], REF_ROW_FRACTION)
-        sample[name] = (np.ascontiguousarray(W[rows]), np.ascontiguousarray(mask[rows]), x[: args.m])
-
     def step():
-        for name in SHAPES:
-            W, mask, x = sample[name]
-            oracle.linear_bf16(x, W, mask)
+        for _ in range(LAYERS):
+            for name in SHAPES:
+                W, mask, x = host[name]
+                oracle.linear_bf16(x[: args.m], W, mask)
 
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         step()
-    t = (time.perf_counter() - t0) / args.steps * REF_ROW_FRACTION * LAYERS
+    t = (time.perf_counter() - t0) / args.steps
     value = args.m / t
     line = {"metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, Llama-2-7B shapes)", "impl": "reference",
-            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
-                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
-                                   f"sparsity, bf16 bitmask format, decode M={args.m}", "M": args.m},
+            "config": {"workload": workload_name(args.pct, args.m), "M": args.m},
             "cpu_baseline": {"value": value, "unit": "tok/s", "cores": cores, "kind": "oracle",
-                             "sample": f"each step: every {REF_ROW_FRACTION}th output row of the four layer-0 "
-                                       f"linears at M={args.m}; time scaled x{REF_ROW_FRACTION * LAYERS}"},
+                             "sample": f"the whole step: {LAYERS} x (qkv, o, gate_up, down) at M={args.m}, "
+                                       f"float64 C oracle, OpenMP over output rows; no extrapolation"},
             "e2e": {"value": value, "unit": "tok/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def workload_name(pct: int, M: int) -> str:
+    return (f"llama2-7b {LAYERS}-layer linear stack (qkv 4096->12288, o 4096->4096, gate_up 4096->22016, "
+            f"down 11008->4096), {pct}% per-row sparsity, bf16 bitmask format, decode M={M}")
 
 
 def chain_bytes(cs, M: int) -> int:
@@ -710,10 +710,9 @@ def run_ours(args):
     workload = f"{dom} {args.pct}% bf16 M={M}"
     roofline = {"bound": "hbm", "achieved": d["gbs"], "peak": peak_gbs, "unit": "GB/s", "frac": d["frac"],
                 "traffic": profiled_traffic(kern, workload), "kernel": kern, "launch": workload,
-                "peak_kind": f"of {peak_kind} (MEASURED_PEAKS.json hbm_gbs, copy)" if peak_kind == "measured"
-                else "of fallback",
+                "peak_kind": f"of {peak_kind}",
                 "algorithmic_bytes_per_launch": d["algorithmic_bytes"], "us_per_launch": d["us_per_launch"],
-                "frac_of_nominal": d["gbs"] / NOMINAL_HBM_GBS, "nominal_gbs": NOMINAL_HBM_GBS}
+                "frac_of_nominal_8tbs": d["gbs"] / NOMINAL_HBM_GBS}
 
     # ---------------------------------------------------------------- end to end
     # Public API calls (no graph), inputs copied from pinned host memory every step and
@@ -766,57 +765,118 @@ def run_ours(args):
     launch_counts = {name: mats[name][0].launch_count(M, args.path) for name in SHAPES}
     del mats
     torch.cuda.empty_cache()
+    sections = {"per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
+                                   "frac_of_peak": v["step_gbs"] / peak_gbs,
+                                   "per_shape": {n: {"us": s["us_per_launch"], "gbs": s["gbs"], "frac": s["frac"]}
+                                                 for n, s in v["per_shape"].items()}}
+                          for m, v in results.items()}}
     host_bf = None
-    if not (args.no_chain and args.no_stack):
+    if world == 1 and not (args.no_chain and args.no_stack):
         from paper_2405_03594_gb300.stack import host_layer as stack_host_layer
 
         host_bf = stack_host_layer(args.pct, False)
-    chained = None if (args.no_chain or world > 1) else chained_section(args, peak_gbs, host_bf)
-    stack = None if (args.no_stack or world > 1) else stack_section(args, peak_gbs, host_bf)
-    prefill = None if (args.no_prefill or world > 1) else prefill_section(args)
-    dense = None if (args.no_dense or world > 1) else dense_section(host, xs, results, Ms)
-    update = None if (args.no_update or world > 1) else update_section(args, host, peak_gbs)
-    sweep = None if (args.no_sweep_config or world > 1) else sweep_section(args, peak_gbs)
+    if world == 1:
+        if not args.no_chain:
+            sections["chained_step_bf16"] = chained_section(args, peak_gbs, host_bf)
+        if not args.no_stack:
+            sections["stack_int8"] = stack_section(args, peak_gbs, host_bf)
+        if not args.no_prefill:
+            sections["prefill"] = prefill_section(args)
+        if not args.no_dense:
+            sections["dense_comparison"] = dense_section(host, xs, results, Ms)
+        if not args.no_update:
+            sections["masked_update"] = update_section(args, host, peak_gbs)
+        if not args.no_sweep_config:
+            sections["sparsity_batch_sweep"] = sweep_section(args, peak_gbs)
 
     if rank == 0:
-        launches_per_step = LAYERS * sum(launch_counts.values())
-        line = {
-            "metric": METRIC, "value": r["tok_s"], "unit": "tok/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic: seeded N(0,0.02^2) bf16 weights, per-row magnitude masks, N(0,1) bf16 x; "
-                    "32 device copies of layer 0",
-            "config": {"workload": f"llama2-7b linear stack, {LAYERS} layers x (qkv 4096->12288, o 4096->4096, "
-                                   f"gate_up 4096->22016, down 11008->4096), {args.pct}% per-row magnitude "
-                                   f"sparsity, bf16 bitmask format, decode M={M}",
-                       "M": M, "layers": LAYERS, "sparsity_pct": args.pct, "path": args.path,
-                       "l2": f"no flush: inputs larger than L2 ({r['step_bytes'] / 1e9:.2f} GB of distinct "
-                             f"compressed weights per step)",
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
-            "e2e": {"value": whole_job_tok_s(world, M, e2e_ms), "unit": "tok/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "how": "public sp.linear calls (no graph) with pinned host x "
-                                                      "copied in and the last down output copied out per step"},
-            "gpu_launches": launches_per_step * args.steps,
-            "roofline": roofline,
-            "cpu_baseline": cpu,
-            "clocks": clocks,
-            "step_gbs": r["step_gbs"],
-            "parity_layer0": parity,
-            "chained_step_bf16": chained,
-            "stack_int8": stack,
-            "prefill": prefill,
-            "dense_comparison": dense,
-            "masked_update": update,
-            "sparsity_batch_sweep": sweep,
-            "per_m": {str(m): {"tok_s": v["tok_s"], "step_ms": v["step_ms"], "step_gbs": v["step_gbs"],
-                               "frac_of_peak": v["step_gbs"] / peak_gbs,
-                               "per_shape": {n: {"us": round(s["us_per_launch"], 3), "gbs": round(s["gbs"], 1),
-                                                 "frac": round(s["frac"], 4)} for n, s in v["per_shape"].items()}}
-                      for m, v in results.items()},
-        }
-        print(json.dumps(line), flush=True)
+        if args.sections_out:
+            with open(args.sections_out, "w") as f:
+                json.dump(sections, f, indent=1)
+        line = headline_line(args, world, r, roofline, {
+            "value": whole_job_tok_s(world, M, e2e_ms), "unit": "tok/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h}, cpu, clocks, parity, LAYERS * sum(launch_counts.values()) * args.steps,
+            section_summary(sections))
+        print(json.dumps(line, separators=(",", ":")), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
+
+
+def _sig(v, n: int = 4):
+    """v rounded to n significant digits (None and non-numbers pass through)."""
+    if isinstance(v, bool) or not isinstance(v, (int, float)):
+        return v
+    if v == 0 or v != v:
+        return v
+    from math import floor, log10
+
+    return round(v, max(0, n - 1 - int(floor(log10(abs(v))))))
+
+
+def section_summary(sections: dict) -> dict:
+    """A few figures of each context section, small enough for the headline line; the
+    full sections go to --sections-out."""
+    out = {}
+    pm = sections.get("per_m") or {}
+    if pm:
+        out["tok_s_by_m"] = {m: _sig(v["tok_s"]) for m, v in pm.items()}
+    ch = sections.get("chained_step_bf16")
+    if ch:
+        out["chain_bf16_tok_s"] = {m: _sig(v["tok_s"]) for m, v in ch.get("chain", {}).items()}
+        out["graph_glue_bf16_tok_s"] = {m: _sig(v["tok_s"]) for m, v in ch.get("graph", {}).items()}
+    st = sections.get("stack_int8")
+    if st:
+        out["stack_int8_tok_s"] = {"graph": {m: _sig(v["tok_s"]) for m, v in st.get("graph_per_m", {}).items()},
+                                   "chain": {m: _sig(v["tok_s"]) for m, v in st.get("chain_per_m", {}).items()}}
+    pf = sections.get("prefill")
+    if pf and pf.get("shapes"):
+        fr = {k: v["frac_dense_executed"] for k, v in pf["shapes"].items()}
+        out["prefill_frac_dense"] = {"min": _sig(min(fr.values()), 3), "max": _sig(max(fr.values()), 3),
+                                     "qkv@70%": _sig(fr.get("qkv@70%"), 3)}
+    up = sections.get("masked_update")
+    if up and up.get("shapes"):
+        out["update_frac"] = {n: _sig(v["frac"], 3) for n, v in up["shapes"].items()}
+    de = sections.get("dense_comparison")
+    if de and de.get("step_speedup"):
+        out["vs_dense_cublas"] = {m: _sig(v, 3) for m, v in de["step_speedup"].items()}
+    sw = sections.get("sparsity_batch_sweep")
+    if sw and sw.get("points"):
+        out["sweep_frac"] = {k: {m: _sig(p["by_m"][m]["frac_of_roofline"], 2) for m in ("1", "16", "64", "256")
+                                 if m in p["by_m"]}
+                             for k, p in sw["points"].items() if k.endswith("@70%")}
+    for k in ("chained_step_bf16", "stack_int8", "prefill", "dense_comparison", "masked_update",
+              "sparsity_batch_sweep"):
+        if sections.get(k) and sections[k].get("error"):
+            out.setdefault("errors", {})[k] = str(sections[k]["error"])[:80]
+    return out
+
+
+def headline_line(args, world: int, r: dict, roofline: dict, e2e: dict, cpu, clocks, parity, gpu_launches: int,
+                  summary: dict) -> dict:
+    """The one JSON line bench.py prints: the contract's keys, the roofline of the dominant
+    kernel, the CPU baseline, the clocks seen while timing, and a compact summary of the
+    context sections (kept to about 2 KB so that the whole line survives a tail capture)."""
+    M = args.m
+    rf = {k: _sig(v) for k, v in roofline.items()}
+    line = {
+        "metric": METRIC, "value": _sig(r["tok_s"], 6), "unit": "tok/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": _sig(r["step_ms"], 6), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded N(0,0.02^2) W, per-row magnitude masks, N(0,1) x; 32 copies of layer 0",
+        "config": {"workload": workload_name(args.pct, M), "M": M, "layers": LAYERS, "sparsity_pct": args.pct,
+                   "path": args.path,
+                   "l2": f"no flush: {r['step_bytes'] / 1e9:.2f} GB of distinct weights per step",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "e2e": {k: _sig(v, 6) for k, v in e2e.items()},
+        "gpu_launches": gpu_launches,
+        "roofline": rf,
+        "cpu_baseline": None if cpu is None else {k: _sig(v) for k, v in cpu.items()},
+        "clocks": clocks,
+        "step_gbs": _sig(r["step_gbs"]),
+        "parity_layer0": None if parity is None else {k: _sig(v, 3) for k, v in parity.items()},
+        "summary": summary,
+    }
+    return line
 
 
 def run_single(args):

@@ -184,3 +184,64 @@ def test_sweep_section_reports_failures_instead_of_raising():
     b = _bench_module()
     out = b.sweep_section(None, 6681.8)
     assert "error" in out and out["points"] == {}
+
+
+def _full_sections():
+    """Context sections shaped like a full run's (every shape, sparsity and batch size)."""
+    per_shape = {n: {"us_per_launch": 24.41234, "gbs": 2680.51234, "frac": 0.401234} for n in ("qkv", "o", "gate_up",
+                                                                                                 "down")}
+    per_m = {str(m): {"tok_s": 445.928809 * m, "step_ms": 2.242510414, "step_gbs": 2095.73218, "frac_of_peak": 0.3136,
+                      "per_shape": {n: {"us": 1.0, "gbs": 2.0, "frac": 0.3} for n in per_shape}} for m in (1, 4, 16)}
+    by_m = {str(m): {"us": 31.5, "tok_s": 1.0, "gbs": 765.97, "tflops_nonzero": 9.15, "bound": "hbm",
+                     "frac_of_roofline": 0.1146353276, "kernel": "linear_tc_kernel"} for m in (1, 2, 4, 8, 16, 32, 64,
+                                                                                               128, 256)}
+    return {
+        "per_m": per_m,
+        "chained_step_bf16": {"chain": {"1": {"tok_s": 420.123456}, "4": {"tok_s": 1229.98765}},
+                              "graph": {"1": {"tok_s": 430.111}, "4": {"tok_s": 1350.222}}},
+        "stack_int8": {"graph_per_m": {"1": {"tok_s": 355.1234}, "16": {"tok_s": 2902.123}, "64": {"tok_s": 9684.1}},
+                       "chain_per_m": {"1": {"tok_s": 368.12}, "4": {"tok_s": 1048.4}}},
+        "prefill": {"shapes": {f"{n}@{p}%": {"frac_dense_executed": 0.3212345} for n in per_shape for p in (50, 70)}},
+        "masked_update": {"shapes": {n: {"frac": 0.4612345} for n in per_shape}},
+        "dense_comparison": {"step_speedup": {"1": 2.3456789, "4": 2.1, "16": 1.9}},
+        "sparsity_batch_sweep": {"points": {f"{n}@{p}%": {"by_m": by_m} for n in ("gate_up", "down")
+                                            for p in (0, 50, 60, 70, 80)}},
+    }
+
+
+def test_headline_line_is_compact_and_complete():
+    """The final stdout line must survive a tail capture whole: about 2 KB at most with
+    every context section present, and carrying every key of the bench contract."""
+    import argparse
+
+    b = _bench_module()
+    args = argparse.Namespace(m=1, pct=70, path="auto", steps=20, warmup=5)
+    r = {"tok_s": 445.92880982, "step_ms": 2.2425104141, "step_gbs": 2095.732184, "step_bytes": 4_700_000_000}
+    roofline = {"bound": "hbm", "achieved": 2680.5123, "peak": 6681.8, "unit": "GB/s", "frac": 0.40116,
+                "traffic": 65_930_000, "kernel": "linear_ccw_kernel", "launch": "gate_up 70% bf16 M=1",
+                "peak_kind": "of measured",
+                "algorithmic_bytes_per_launch": 65_440_000, "us_per_launch": 24.41234,
+                "frac_of_nominal_8tbs": 0.3350123}
+    e2e = {"value": 422.123456789, "unit": "tok/s", "h2d_bytes_per_step": 8192 * 4 + 22016, "d2h_bytes_per_step": 8192}
+    cpu = {"value": 1.1812345, "unit": "tok/s", "cores": 16, "kind": "oracle",
+           "sample": "layer 0 (qkv, o, gate_up, down) at M=1, float64 C oracle, OpenMP over rows; "
+                     "median of 12 runs of 0.85 s, x32 layers"}
+    clocks = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 123}
+    parity = {"max_err_over_max_ref": 0.00212345, "rel_fro": 0.00112345, "ok": True}
+    line = b.headline_line(args, 1, r, roofline, e2e, cpu, clocks, parity, 20 * 128,
+                           b.section_summary(_full_sections()))
+    text = json.dumps(line, separators=(",", ":"))  # as bench.py prints it
+    assert len(text) <= 2048, len(text)
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "config", "e2e", "gpu_launches", "roofline", "cpu_baseline", "clocks"):
+        assert k in line, k
+    assert line["config"]["workload"] and line["roofline"]["frac"] == pytest.approx(0.4012, abs=1e-4)
+    assert line["value"] == pytest.approx(445.929, rel=1e-5)
+    assert set(line["summary"]["sweep_frac"]) == {"gate_up@70%", "down@70%"}
+    assert "errors" not in line["summary"]
+
+
+def test_section_summary_reports_section_errors():
+    b = _bench_module()
+    s = b.section_summary({"prefill": {"error": "RuntimeError: " + "x" * 500, "shapes": {}}})
+    assert s["errors"]["prefill"].startswith("RuntimeError") and len(s["errors"]["prefill"]) <= 80
