@@ -175,7 +175,11 @@ sp_status sp_linear_noalloc(const sp_matrix* h, const void* x_dev, int64_t m, vo
  *              unchanged.
  * bf16 handles only (SP_ERR_UNSUPPORTED for SP_INT8).  Asynchronous on `stream`; work
  * that reads the handle (sp_linear, sp_decompress, ...) must be ordered after it by the
- * caller.  No allocation, no host sync.  Results are bitwise deterministic. */
+ * caller, on the same stream or through an event.  The next sp_linear launch on the
+ * handle then starts only once the update has finished (it is launched without
+ * programmatic dependent launch, whose early start would let its first weight copies
+ * read the values from before the update).  No allocation, no host sync.  Results are
+ * bitwise deterministic. */
 sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float lr, void* stream);
 
 /* INT8 weights and INT8 activations (Sec. 3.4, the sparse INT8 deployment):

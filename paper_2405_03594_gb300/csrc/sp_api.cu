@@ -179,6 +179,7 @@ sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, vo
   c->d_off = nullptr;
   c->d_qidx = nullptr;
   c->d_scale = nullptr;
+  c->weights_written = 0;  // the copy below is synchronised
   const size_t off_bytes = ((size_t)h->RB * h->T + 1) * sizeof(uint64_t);
   cudaStream_t s = (cudaStream_t)stream;
   sp_status st = SP_OK;

@@ -31,6 +31,11 @@ struct sp_matrix {
   void* ctx;
   int32_t device;
   int32_t num_sms;
+  // Set by sp_masked_update, which rewrites d_buf in place; cleared by the next linear
+  // launch on this handle, which then goes without programmatic dependent launch: the
+  // decode kernels copy their first weight chunks before griddepcontrol.wait, and only
+  // that wait makes the previous grid's writes visible.
+  mutable int32_t weights_written;
 };
 
 namespace sp {

@@ -620,7 +620,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
 
 // kind 0: thread-per-row kernel; kind 1: warp-per-chunk kernel (M <= 4)
 template <int M, int ES>
-sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind) {
+sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, bool pdl) {
   void (*kern)(const LinearParams);
   if constexpr (M <= 4) {
     if (kind == 1)
@@ -650,7 +650,7 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, in
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   int na = 1;
   if (p.cluster > 1) {
     attr[1].id = cudaLaunchAttributeClusterDimension;
@@ -669,24 +669,24 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, in
 }
 
 template <int ES>
-sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, int kind) {
+sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, bool pdl) {
   switch (p.M) {
-    case 1: return launch_one<1, ES>(p, stream, smem, kind);
-    case 2: return launch_one<2, ES>(p, stream, smem, kind);
-    case 3: return launch_one<3, ES>(p, stream, smem, kind);
-    case 4: return launch_one<4, ES>(p, stream, smem, kind);
-    case 5: return launch_one<5, ES>(p, stream, smem, kind);
-    case 6: return launch_one<6, ES>(p, stream, smem, kind);
-    case 7: return launch_one<7, ES>(p, stream, smem, kind);
-    case 8: return launch_one<8, ES>(p, stream, smem, kind);
-    case 9: return launch_one<9, ES>(p, stream, smem, kind);
-    case 10: return launch_one<10, ES>(p, stream, smem, kind);
-    case 11: return launch_one<11, ES>(p, stream, smem, kind);
-    case 12: return launch_one<12, ES>(p, stream, smem, kind);
-    case 13: return launch_one<13, ES>(p, stream, smem, kind);
-    case 14: return launch_one<14, ES>(p, stream, smem, kind);
-    case 15: return launch_one<15, ES>(p, stream, smem, kind);
-    case 16: return launch_one<16, ES>(p, stream, smem, kind);
+    case 1: return launch_one<1, ES>(p, stream, smem, kind, pdl);
+    case 2: return launch_one<2, ES>(p, stream, smem, kind, pdl);
+    case 3: return launch_one<3, ES>(p, stream, smem, kind, pdl);
+    case 4: return launch_one<4, ES>(p, stream, smem, kind, pdl);
+    case 5: return launch_one<5, ES>(p, stream, smem, kind, pdl);
+    case 6: return launch_one<6, ES>(p, stream, smem, kind, pdl);
+    case 7: return launch_one<7, ES>(p, stream, smem, kind, pdl);
+    case 8: return launch_one<8, ES>(p, stream, smem, kind, pdl);
+    case 9: return launch_one<9, ES>(p, stream, smem, kind, pdl);
+    case 10: return launch_one<10, ES>(p, stream, smem, kind, pdl);
+    case 11: return launch_one<11, ES>(p, stream, smem, kind, pdl);
+    case 12: return launch_one<12, ES>(p, stream, smem, kind, pdl);
+    case 13: return launch_one<13, ES>(p, stream, smem, kind, pdl);
+    case 14: return launch_one<14, ES>(p, stream, smem, kind, pdl);
+    case 15: return launch_one<15, ES>(p, stream, smem, kind, pdl);
+    case 16: return launch_one<16, ES>(p, stream, smem, kind, pdl);
     default: return SP_ERR_INVALID_ARG;
   }
 }
@@ -795,9 +795,13 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.part_off = pl.part_off;
     const int kind = pl.kind;
     const size_t smem = pl.smem;
+    // after an in-place weight update the first launch waits for the whole previous grid
+    // (no weight copy may start before its writes are visible)
+    const bool pdl = !(m0 == 0 && h->weights_written);
     const sp_status st =
-        h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind) : dispatch_m<1>(p, stream, smem, kind);
+        h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind, pdl) : dispatch_m<1>(p, stream, smem, kind, pdl);
     if (st != SP_OK) return st;
+    h->weights_written = 0;
   }
   return SP_OK;
 }

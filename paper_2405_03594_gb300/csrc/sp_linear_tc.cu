@@ -633,7 +633,7 @@ int ntok_for(int64_t M) {
 
 template <int ES>
 sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtensorMap& map_y, size_t smem,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, bool pdl) {
   auto kern = linear_tc_kernel<ES>;
   static bool configured[kMaxDevices] = {};
   int dev = 0;
@@ -653,7 +653,7 @@ sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtenso
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   if (cudaLaunchKernelEx(&cfg, kern, tp, map, map_y) != cudaSuccess) {
@@ -748,8 +748,13 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return SP_ERR_CUDA;
   }
-  return h->esize == 2 ? launch_tc_es<2>(tp, map, map_y, smem, stream)
-                       : launch_tc_es<1>(tp, map, map_y, smem, stream);
+  // after an in-place weight update the launch waits for the whole previous grid (no
+  // weight copy may start before its writes are visible)
+  const bool pdl = !h->weights_written;
+  st = h->esize == 2 ? launch_tc_es<2>(tp, map, map_y, smem, stream, pdl)
+                     : launch_tc_es<1>(tp, map, map_y, smem, stream, pdl);
+  if (st == SP_OK) h->weights_written = 0;
+  return st;
 }
 
 }  // namespace sp

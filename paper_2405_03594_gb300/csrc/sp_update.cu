@@ -132,5 +132,6 @@ extern "C" sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float
   masked_update_kernel<<<(unsigned)C, kUpdThreads, 0, (cudaStream_t)stream>>>(h->d_buf, h->d_off, grad_dev, -lr, h->N,
                                                                           h->K, h->T);
   if (cudaGetLastError() != cudaSuccess) return SP_ERR_CUDA;
+  h->weights_written = 1;
   return SP_OK;
 }

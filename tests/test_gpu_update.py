@@ -105,6 +105,36 @@ def test_updated_handle_runs_linear(sp, oracle):
     gu.assert_close(gu.bf16_from_dev(y), oracle.linear_bf16(x, Wn, mask), "linear after update")
 
 
+@pytest.mark.parametrize("M,path", [(1, "cuda_core"), (4, "cuda_core"), (32, "tensor_core")])
+def test_update_then_linear_on_one_stream_without_host_sync(sp, oracle, M, path):
+    """Steps and products queued back to back on one stream, the host never waiting in
+    between: each product must see the weights of the step just before it.  (The decode
+    kernels copy their first weight chunks before waiting on the previous grid, so the
+    launch right after an in-place update has to wait for it in full.)  A large step size
+    makes a stale read show in the outputs."""
+    import torch
+
+    N, K = 4096, 4096
+    W, mask, grad = _case(N, K, 70, 31)
+    x = synth.activations(M, K, np.random.default_rng(5))
+    h = sp.compress(gu.bf16_to_dev(W), gu.u8_to_dev(mask))
+    xd, gd = gu.bf16_to_dev(x), gu.f32_to_dev(grad)
+    ws = torch.zeros(max(h.workspace_size(M), 256), dtype=torch.uint8, device=gu.dev())
+    torch.cuda.synchronize()
+    ys = []
+    for _ in range(3):
+        h.masked_update(gd, 0.5)
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=gu.dev())
+        h.linear(xd, out=y, workspace=ws, path=path)
+        ys.append(y)
+    sp.check()
+    buf, off = oracle.compress(W, mask)
+    for i, y in enumerate(ys):
+        buf = oracle.masked_update_bf16(buf, off, N, K, grad, 0.5)
+        Wi = oracle.decompress(buf, off, N, K, np.uint16)
+        gu.assert_close(gu.bf16_from_dev(y), oracle.linear_bf16(x, Wi, mask), f"product after step {i + 1}")
+
+
 def test_gate_up_shape_70pct(sp, oracle):
     """The largest Llama-2-7B shape (gate/up 22016 x 4096) at 70 %: every updated byte."""
     name = "gate_up"
