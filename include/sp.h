@@ -158,6 +158,8 @@ sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* 
  *   Returns SP_ERR_WORKSPACE if the kernel would need more scratch than the array holds.
  *   The first call on a device looks up the array's device address (set-up, once per
  *   device, with that device current); make that first call before any stream capture.
+ *   The address is kept for the life of the process, so a device reset (cudaDeviceReset)
+ *   between calls is not supported.
  *   Every call on a device shares the one array, and a call clears its arrival counters
  *   first: calls that overlap on the GPU (other streams, other threads) race and give
  *   wrong results; order them on one stream. */
@@ -203,6 +205,21 @@ sp_status sp_linear_w8a8(const sp_matrix* h, const int8_t* qx_dev, const float* 
 /* Workspace bytes sp_linear_w8a8 needs for a batch of m rows (0 for m == 0).  Host only.
  * SP_ERR_INVALID_ARG for m < 0 or a null `bytes`, SP_ERR_BAD_HANDLE for a dead handle. */
 sp_status sp_w8a8_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
+
+/* Failure-path test (the paper has no counterpart; nothing calls it in normal use).  Runs
+ * sp_linear's CUDA-core decode kernel for m = 1..4 rows -- the warp-per-chunk kernel, as
+ * sp_linear would -- with one consumer warp of its first CTA first waiting on a
+ * shared-memory barrier that nothing completes and no copy targets.  That bounded wait gives
+ * up after wait_ms milliseconds and records SP_ERR_TIMEOUT in the device status word, as any
+ * expired wait does; the warp then goes on normally, so the launch ends and y is the product
+ * sp_linear would give.  Afterwards sp_check() returns SP_ERR_TIMEOUT once (and clears the
+ * status), and the workspace is ready for the next call.  Arguments as for sp_linear;
+ * wait_ms in 1..10000 (SP_ERR_INVALID_ARG otherwise); SP_ERR_UNSUPPORTED when m is outside
+ * 1..4, for an SP_INT8 handle, or when sp_linear would not run the warp-per-chunk kernel
+ * for this matrix.  The waiting warp is compiled into a variant of the kernel of its own;
+ * sp_linear never runs that variant. */
+sp_status sp_test_expired_wait(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
+                               size_t workspace_bytes, uint32_t wait_ms, void* stream);
 
 /* A copy of the handle with its own device buffers (same bytes), allocated on the
  * current device, which must be the handle's (SP_ERR_INVALID_ARG otherwise).  The copies

@@ -158,6 +158,24 @@ sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_de
   return sp_linear_ex(h, x_dev, m, y_dev, workspace_dev, workspace_bytes, SP_PATH_AUTO, stream);
 }
 
+sp_status sp_test_expired_wait(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
+                               size_t workspace_bytes, uint32_t wait_ms, void* stream) {
+  if (!live(h)) return SP_ERR_BAD_HANDLE;
+  if (!x_dev || !y_dev || wait_ms < 1 || wait_ms > 10000) return SP_ERR_INVALID_ARG;
+  if (m < 1 || m > 4 || h->esize != 2 || cc_kernel_kind(h, m) != 1) return SP_ERR_UNSUPPORTED;
+  if (!aligned16(x_dev) || !aligned16(y_dev) || (workspace_dev && !aligned16(workspace_dev))) return SP_ERR_ALIGNMENT;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
+  if (dev != h->device) return SP_ERR_INVALID_ARG;
+  if (!workspace_dev || workspace_bytes < std::max(workspace_bytes_cc(h, m), workspace_bytes_tc(h, m)))
+    return SP_ERR_WORKSPACE;
+  return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
+                          workspace_bytes, (cudaStream_t)stream, true, (uint64_t)wait_ms * 1000000ull);
+}
+
 sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx, void* stream,
                    sp_matrix** out) {
   if (!out) return SP_ERR_INVALID_ARG;

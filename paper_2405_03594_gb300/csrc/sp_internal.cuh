@@ -76,6 +76,8 @@ struct LinearParams {
                         // one thread-block cluster; <= 1 = stream-K over the workspace
   uint32_t part_off;    // cluster mode: shared-memory offset of the CTA's FP32 partial
   uint32_t comb_off;    // warp-per-chunk kernel: shared-memory offset of the warps' partials
+  uint64_t probe_ns;    // 0, except in the failure-path test: consumer warp 0 of CTA 0 first
+                        // waits this long on a barrier that nothing completes
 };
 
 // Workspace layout, fixed per device so that calls with different grids can share it:
@@ -256,7 +258,7 @@ sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream
 // allow_cluster: split small row-block counts over thread-block clusters (no workspace
 // needed); otherwise stream-K with split-K partials in the workspace.
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream, bool allow_cluster = true);
+                           cudaStream_t stream, bool allow_cluster = true, uint64_t probe_ns = 0);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
 int cc_kernel_kind(const sp_matrix* h, int64_t M);  // 0 thread-per-row, 1 warp-per-chunk, -1 none fits
 sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,

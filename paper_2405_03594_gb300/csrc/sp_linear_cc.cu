@@ -485,7 +485,7 @@ __device__ __forceinline__ void flush_async(const LinearParams& p, FlushCtl* ctl
 // order (deterministic): in stream-K mode by the last warp to get there, which runs the
 // row block's end alone while the others go on (flush_async); in cluster mode, where a
 // CTA's one row block ends with its range, by thread r <-> row r after a barrier.
-template <int M, int ES, bool CL>
+template <int M, int ES, bool CL, bool PROBE = false>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -495,6 +495,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
   volatile int* tag = s_flag + 4;
   float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [2][kConsumerWarps][M][kRows]
   FlushCtl* fctl = reinterpret_cast<FlushCtl*>(comb + 2 * kConsumerWarps * M * kRows);
+  // PROBE (the failure-path test only): a barrier that nothing completes, in the unused upper
+  // half of the 16-byte flag area (8-byte aligned: it follows the mbarrier arrays)
+  uint64_t* probe = reinterpret_cast<uint64_t*>(const_cast<int*>(s_flag) + 2);
   const int T = p.T;
   const int slots = p.slots;  // >= kConsumerWarps
   int64_t w0, w1;
@@ -511,6 +514,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
       fctl->flushed[b] = 0;
       fctl->ready[b] = b;
     }
+    if constexpr (PROBE) mbar_init(probe, 1);
     fence_barrier_init();
   }
   __syncthreads();
@@ -523,6 +527,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
   pdl_wait();
   pdl_launch_dependents();
   bool dead = false;
+  if (PROBE && blockIdx.x == 0 && warp == 0) {
+    // failure-path test: a bounded wait on a barrier that nothing completes and no copy
+    // targets; its expiry is recorded in the status word like any other, and the warp then
+    // goes on normally (every copy it consumes has landed, so the results stay correct)
+    if (!__all_sync(0xffffffffu, mbar_wait(probe, 0, p.probe_ns))) set_status(p.status, kStatusTimeout);
+  }
   int s = warp;  // ring slot of this warp's next item (item n uses slot n % slots)
   uint32_t ph = 0;
   int64_t w = w0 + warp;
@@ -623,25 +633,31 @@ template <int M, int ES>
 sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, bool pdl) {
   void (*kern)(const LinearParams);
   if constexpr (M <= 4) {
-    if (kind == 1)
+    if (kind == 1 && p.probe_ns != 0) {
+      if constexpr (ES == 2)
+        kern = p.cluster > 1 ? linear_ccw_kernel<M, ES, true, true> : linear_ccw_kernel<M, ES, false, true>;
+      else
+        return SP_ERR_UNSUPPORTED;
+    } else if (kind == 1)
       kern = p.cluster > 1 ? linear_ccw_kernel<M, ES, true> : linear_ccw_kernel<M, ES, false>;
     else
       kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
   } else {
     kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
   }
-  static bool configured[2][2][kMaxDevices] = {};  // kernel attributes, once per device
+  static bool configured[3][2][kMaxDevices] = {};  // kernel attributes, once per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
   const int ci = p.cluster > 1 ? 1 : 0;
-  if (!configured[kind][ci][dev]) {
+  const int ki = p.probe_ns != 0 ? 2 : kind;  // the probe variant is a kernel of its own
+  if (!configured[ki][ci][dev]) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess ||
         (ci && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
       cudaGetLastError();
       return SP_ERR_CUDA;
     }
-    configured[kind][ci][dev] = true;
+    configured[ki][ci][dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)p.G);
@@ -762,7 +778,7 @@ size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
 }
 
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream, bool allow_cluster) {
+                           cudaStream_t stream, bool allow_cluster, uint64_t probe_ns) {
   const int S = allow_cluster ? cluster_cc(h) : 1;
   const size_t need = workspace_bytes_cc(h, M);
   if (S == 1 && (!ws || ws_bytes < need)) return SP_ERR_WORKSPACE;
@@ -781,6 +797,7 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.cnt = reinterpret_cast<int*>(ws);
   p.ws = ws ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms)) : nullptr;
   p.timeout_ns = wait_timeout_ns();
+  p.probe_ns = probe_ns;
   p.chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
   for (int64_t m0 = 0; m0 < M; m0 += kMaxTokens) {
     const int Mt = (int)std::min<int64_t>(kMaxTokens, M - m0);

@@ -25,7 +25,7 @@ STATUS = {
 }
 # every function declared in include/sp.h and include/sp_stack.h
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
-           "sp_linear_noalloc", "sp_masked_update", "sp_linear_w8a8", "sp_w8a8_workspace_size",
+           "sp_linear_noalloc", "sp_test_expired_wait", "sp_masked_update", "sp_linear_w8a8", "sp_w8a8_workspace_size",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
            "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_chain_workspace_size", "sp_chain_run"]
 
@@ -70,6 +70,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_linear.argtypes = [P, P, I64, P, P, SZ, P]
     lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
     lib.sp_linear_noalloc.argtypes = [P, P, I64, P, P]
+    lib.sp_test_expired_wait.argtypes = [P, P, I64, P, P, SZ, ctypes.c_uint32, P]
     lib.sp_masked_update.argtypes = [P, P, ctypes.c_float, P]
     lib.sp_linear_w8a8.argtypes = [P, P, P, I64, P, P, SZ, P]
     lib.sp_w8a8_workspace_size.argtypes = [P, I64, ctypes.POINTER(SZ)]
@@ -95,7 +96,9 @@ _lib = load_library()
 
 # ------------------------------------------------------------------ torch-backed allocator
 _live = {}
-_live_lock = threading.Lock()
+# re-entrant: a handle collected while this thread holds the lock (its __del__ frees buffers
+# through _free) must not deadlock
+_live_lock = threading.RLock()
 
 
 def _alloc(nbytes, ctx):
@@ -189,6 +192,15 @@ class SparseMatrix:
         assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
         _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)), "sp_linear_noalloc")
         return out
+
+    def test_expired_wait(self, x: torch.Tensor, out: torch.Tensor, workspace: torch.Tensor, wait_ms: int,
+                          stream=None) -> None:
+        """sp_test_expired_wait: the decode kernel with one warp's bounded wait made to expire
+        (the failure-path test); sp.check() afterwards raises SP_ERR_TIMEOUT."""
+        assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
+        assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
+        _check(_lib.sp_test_expired_wait(self._h, _ptr(x), x.shape[0], _ptr(out), _ptr(workspace), workspace.numel(),
+                                         wait_ms, _stream(stream)), "sp_test_expired_wait")
 
     def w8a8_workspace_size(self, m: int) -> int:
         b = ctypes.c_size_t()
