@@ -10,8 +10,9 @@ Per layer, four fused sparse linears and the elementwise glue of include/sp_stac
     h   = h + a.Wdown^T + r'_l                  (sparse linear, sp_residual_add)
 
 All arithmetic runs in libsp kernels; PyTorch only holds the buffers.  The layers are
-device copies of one seeded layer (each its own HBM buffers), so a step streams the
-full 32-layer weight set.  `capture()` records one step as a single CUDA graph.
+device copies of one seeded layer (each its own HBM buffers, so a step streams the full
+32-layer weight set), or each layer's own seeded inputs (`host_layers`: distinct weights,
+or a per-layer sparsity profile).  `capture()` records one step as a single CUDA graph.
 
 `ChainStack` runs the same step (for batches of up to 4 rows) as one persistent launch of
 sp_chain_run: the glue is fused into the linears' epilogues (v is read in place from
@@ -35,38 +36,53 @@ D_FF = 11008
 STACK_WEIGHT_STD = 0.003
 
 
-def host_layer(pct: int, int8: bool, seed: int = 0, std: float = STACK_WEIGHT_STD):
+def host_layer(pct, int8: bool, seed: int = 0, std: float = STACK_WEIGHT_STD, layer: int = 0):
     """Seeded host inputs of one layer: {shape: (values, mask, scale or None)}."""
+    return synth.stack_layer(pct, int8, seed=seed, layer=layer, std=std)
+
+
+def _compress_layer(host: dict, dev, interleave_gate_up: bool = False) -> dict:
+    """{shape: SparseMatrix} of one layer's host inputs (gate/up rows interleaved for the
+    chained step's pair epilogue)."""
     out = {}
     for name in SHAPES:
-        N, K = synth.LLAMA2_7B_SHAPES[name]
-        p = synth.PROJ_IDS[name]
-        W = synth.weight(N, K, synth.rng(seed, 0, p, synth.STREAM_W), std=std)
-        mask = synth.magnitude_mask(W, pct)
-        if int8:
-            q, s = synth.quantize_int8(W, mask)
-            out[name] = (q, mask, s)
+        vals, mask, s = host[name]
+        if interleave_gate_up and name == "gate_up":
+            vals, mask = interleave_rows(vals, D_FF), interleave_rows(mask, D_FF)
+            s = None if s is None else interleave_rows(s, D_FF)
+        vals, mask = np.ascontiguousarray(vals), np.ascontiguousarray(mask)
+        if s is not None:
+            out[name] = sp.compress(torch.from_numpy(vals).to(dev), torch.from_numpy(mask).to(dev),
+                                    torch.from_numpy(np.ascontiguousarray(s)).to(dev))
         else:
-            out[name] = (W, mask, None)
+            out[name] = sp.compress(torch.from_numpy(vals.view(np.int16)).to(dev).view(torch.bfloat16),
+                                    torch.from_numpy(mask).to(dev))
     return out
 
 
+def _layer_mats(layers: int, host, host_layers, dev, interleave_gate_up: bool) -> dict:
+    """{shape: [SparseMatrix per layer]}: device copies of one layer (host), or each layer's
+    own inputs (host_layers, one dict per layer)."""
+    if host_layers is not None:
+        per = [_compress_layer(hl, dev, interleave_gate_up) for hl in host_layers]
+        return {name: [p[name] for p in per] for name in SHAPES}
+    one = _compress_layer(host, dev, interleave_gate_up)
+    return {name: [one[name]] + [one[name].clone() for _ in range(layers - 1)] for name in SHAPES}
+
+
 class LinearStack:
+    """host: one layer's inputs, copied to every layer; host_layers: each layer's own inputs
+    (then `layers` is their count)."""
+
     def __init__(self, layers: int = 32, pct: int = 70, int8: bool = True, max_m: int = 64, seed: int = 0,
-                 device=None, host=None, path: str = "auto"):
+                 device=None, host=None, path: str = "auto", host_layers=None):
         self.dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+        if host_layers is not None:
+            layers = len(host_layers)
         self.layers, self.max_m, self.path = layers, max_m, path
-        self.host = host_layer(pct, int8, seed) if host is None else host
-        self.mats = {}
-        for name in SHAPES:
-            vals, mask, s = self.host[name]
-            if s is not None:
-                h0 = sp.compress(torch.from_numpy(vals).to(self.dev), torch.from_numpy(mask).to(self.dev),
-                                 torch.from_numpy(s).to(self.dev))
-            else:
-                h0 = sp.compress(torch.from_numpy(vals.view(np.int16)).to(self.dev).view(torch.bfloat16),
-                                 torch.from_numpy(mask).to(self.dev))
-            self.mats[name] = [h0] + [h0.clone() for _ in range(layers - 1)]
+        self.host = None if host_layers is not None else (host_layer(pct, int8, seed) if host is None else host)
+        self.host_layers = host_layers
+        self.mats = _layer_mats(layers, self.host, host_layers, self.dev, False)
         g = synth.rng(seed, 0, 9, synth.STREAM_RESID)
         r = synth.activations(2 * layers, D_MODEL, g)
         rt = torch.from_numpy(r.view(np.int16)).to(self.dev).view(torch.bfloat16)
@@ -86,8 +102,11 @@ class LinearStack:
         torch.cuda.synchronize()
 
     def weight_bytes(self) -> int:
-        return self.layers * sum(int(self.mats[n][0].info.bytes) + int(self.mats[n][0].info.scale_bytes)
-                                 for n in SHAPES)
+        return sum(int(m.info.bytes) + int(m.info.scale_bytes) for n in SHAPES for m in self.mats[n])
+
+    def host_of(self, layer: int, name: str):
+        """Host (values, mask, scale) of `name` in `layer`."""
+        return (self.host_layers[layer] if self.host_layers is not None else self.host)[name]
 
     def launches_per_step(self, M: int, reset: bool = True) -> int:
         """libsp kernels per step: the four sparse linears (as many launches as the library
@@ -150,24 +169,14 @@ class ChainStack:
     """The 32-layer linear stack as one sp_chain_run call per decode step (m <= 4 rows)."""
 
     def __init__(self, layers: int = 32, pct: int = 70, int8: bool = False, max_m: int = 4, seed: int = 0,
-                 device=None, host=None):
+                 device=None, host=None, host_layers=None):
         self.dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+        if host_layers is not None:
+            layers = len(host_layers)
         self.layers, self.max_m = layers, max_m
-        self.host = host_layer(pct, int8, seed) if host is None else host
-        self.mats = {}
-        for name in SHAPES:
-            vals, mask, s = self.host[name]
-            if name == "gate_up":
-                vals, mask = interleave_rows(vals, D_FF), interleave_rows(mask, D_FF)
-                s = None if s is None else interleave_rows(s, D_FF)
-            if s is not None:
-                h0 = sp.compress(torch.from_numpy(np.ascontiguousarray(vals)).to(self.dev),
-                                 torch.from_numpy(np.ascontiguousarray(mask)).to(self.dev),
-                                 torch.from_numpy(np.ascontiguousarray(s)).to(self.dev))
-            else:
-                h0 = sp.compress(torch.from_numpy(np.ascontiguousarray(vals).view(np.int16)).to(self.dev)
-                                 .view(torch.bfloat16), torch.from_numpy(np.ascontiguousarray(mask)).to(self.dev))
-            self.mats[name] = [h0] + [h0.clone() for _ in range(layers - 1)]
+        self.host = None if host_layers is not None else (host_layer(pct, int8, seed) if host is None else host)
+        self.host_layers = host_layers
+        self.mats = _layer_mats(layers, self.host, host_layers, self.dev, True)
         g = synth.rng(seed, 0, 9, synth.STREAM_RESID)
         r = synth.activations(2 * layers, D_MODEL, g)
         rt = torch.from_numpy(r.view(np.int16)).to(self.dev).view(torch.bfloat16)
@@ -182,8 +191,16 @@ class ChainStack:
         torch.cuda.synchronize()
 
     def weight_bytes(self) -> int:
-        return self.layers * sum(int(self.mats[n][0].info.bytes) + int(self.mats[n][0].info.scale_bytes)
-                                 for n in SHAPES)
+        return sum(int(m.info.bytes) + int(m.info.scale_bytes) for n in SHAPES for m in self.mats[n])
+
+    def host_of(self, layer: int, name: str):
+        """Host (values, mask, scale) of `name` in `layer`, in the stored row order (gate/up
+        interleaved)."""
+        vals, mask, s = (self.host_layers[layer] if self.host_layers is not None else self.host)[name]
+        if name == "gate_up":
+            vals, mask = interleave_rows(vals, D_FF), interleave_rows(mask, D_FF)
+            s = None if s is None else interleave_rows(s, D_FF)
+        return vals, mask, s
 
     def ops(self, M: int):
         """The chain of one decode step: four linears per layer."""

@@ -149,12 +149,22 @@ def nonuniform_mask(W: np.ndarray, pct: int, g: np.random.Generator):
 
 
 def quantize_int8(W: np.ndarray, mask: np.ndarray):
-    """(q int8 [N, K], s float32 [N]) by symmetric absmax over the kept weights."""
-    w = bf16_to_f32(W).astype(np.float64) * (mask != 0)
-    amax = np.abs(w).max(axis=1)
-    s = np.where(amax > 0, amax / 127.0, 1.0).astype(np.float32)
-    q = np.clip(np.rint(w / s.astype(np.float64)[:, None]), -127, 127).astype(np.int8)
-    q[mask == 0] = 0
+    """(q int8 [N, K], s float32 [N]) by symmetric absmax over the kept weights (row blocks
+    at a time; every element's arithmetic is the same as on the whole matrix)."""
+    N, K = W.shape
+    q = np.empty((N, K), dtype=np.int8)
+    s = np.empty(N, dtype=np.float32)
+    rows = max(1, (1 << 18) // max(K, 1))
+    for r0 in range(0, N, rows):
+        r1 = min(N, r0 + rows)
+        keep = mask[r0:r1] != 0
+        w = bf16_to_f32(W[r0:r1]).astype(np.float64) * keep
+        amax = np.abs(w).max(axis=1)
+        sr = np.where(amax > 0, amax / 127.0, 1.0).astype(np.float32)
+        qq = np.clip(np.rint(w / sr.astype(np.float64)[:, None]), -127, 127).astype(np.int8)
+        qq[~keep] = 0
+        q[r0:r1] = qq
+        s[r0:r1] = sr
     return q, s
 
 
@@ -166,6 +176,43 @@ def quantize_activations_int8(x: np.ndarray):
     sx = np.where(amax > 0, amax / 127.0, 1.0).astype(np.float32)
     qx = np.clip(np.rint(xf / sx.astype(np.float64)[:, None]), -127, 127).astype(np.int8)
     return qx, sx
+
+
+# The four fused linears of one Llama-2-7B layer, in the order a decode step runs them.
+STACK_SHAPES = ("qkv", "o", "gate_up", "down")
+
+
+def stack_layer(pct, int8: bool, seed: int = 0, layer: int = 0, std: float = 0.02) -> dict:
+    """Seeded host inputs of one layer of the linear stack: {shape: (values, mask, scale or
+    None)} with W ~ N(0, std^2) drawn from rng(seed, layer, proj, STREAM_W), per-row magnitude
+    masks at `pct` percent (one int for every shape, or {shape: pct}), and for INT8 the
+    absmax (q, s) pair."""
+    out = {}
+    for name in STACK_SHAPES:
+        N, K = LLAMA2_7B_SHAPES[name]
+        W = weight(N, K, rng(seed, layer, PROJ_IDS[name], STREAM_W), std=std)
+        mask = magnitude_mask(W, pct[name] if isinstance(pct, dict) else pct)
+        if int8:
+            q, s = quantize_int8(W, mask)
+            out[name] = (q, mask, s)
+        else:
+            out[name] = (W, mask, None)
+    return out
+
+
+def layer_sparsity_profile(layers: int, mean: int = 70, spread: int = 10, seed: int = 0) -> list:
+    """A per-layer sparsity profile (percent per layer) standing in for an outlier-weighted
+    layerwise profile: five levels mean - spread, mean - spread/2, mean, mean + spread/2,
+    mean + spread in counts symmetric about the mean (so the profile's mean is exactly
+    `mean`), assigned to layers by a seeded permutation."""
+    lv = [mean - spread, mean - spread // 2, mean, mean + spread // 2, mean + spread]
+    edge = layers // 8
+    half = (layers - 2 * edge) // 2 - (layers - 2 * edge) // 6
+    mid = layers - 2 * edge - 2 * half
+    counts = [edge, half, mid, half, edge]
+    prof = [v for v, c in zip(lv, counts) for _ in range(c)]
+    order = rng(seed, 0, 11, STREAM_MASK).permutation(layers)
+    return [int(prof[i]) for i in order]
 
 
 def layer_inputs(shape_name: str, pct: int, M: int, seed: int = 0, layer: int = 0):

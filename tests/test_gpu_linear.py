@@ -205,6 +205,13 @@ def test_config_prefill_2048_sampled(sp, oracle, name, pct):
 
     got = gu.bf16_from_dev(y[:, torch.from_numpy(rows).to(y.device)])
     gu.assert_close(got, ref, f"prefill {name} {pct}% M=2048")
+    # every output row for eight tokens (first, last, six random): every row block, every
+    # stream-K fix-up and every TMA-store tile of the launch
+    toks = np.sort(np.random.default_rng(pct * 7 + N).choice(np.arange(1, 2047), 6, replace=False))
+    toks = np.concatenate([[0], toks, [2047]])
+    ref_t = oracle.linear_bf16(np.ascontiguousarray(x[toks]), W, mask)
+    got_t = gu.bf16_from_dev(y[torch.from_numpy(toks).to(y.device)])
+    gu.assert_close(got_t, ref_t, f"prefill {name} {pct}% M=2048, all rows of tokens {toks.tolist()}")
 
 
 @pytest.mark.parametrize("name", ["gate_up", "down"])
@@ -222,9 +229,21 @@ def test_config_sweep_nonuniform_sampled(sp, oracle, name, pct):
     rows = np.sort(np.random.default_rng(pct).choice(N, 192, replace=False))
     rows[0], rows[-1] = 0, N - 1
     ref = oracle.linear_bf16(x, W[rows], mask[rows])
+    # every output row for a few tokens of each batch size (all tokens up to M = 8; else the
+    # first, the last and six random ones); the oracle runs once on the union of those tokens
+    rng = np.random.default_rng(pct + 11)
+    toks_by_m = {}
+    for M in (1, 2, 4, 8, 16, 32, 64, 128, 256):
+        toks_by_m[M] = (np.arange(M) if M <= 8 else
+                        np.concatenate([[0], np.sort(rng.choice(np.arange(1, M - 1), 6, replace=False)), [M - 1]]))
+    union = np.unique(np.concatenate(list(toks_by_m.values())))
+    ref_u = oracle.linear_bf16(np.ascontiguousarray(x[union]), W, mask)
+    pos = {int(tk): i for i, tk in enumerate(union)}
     for M in (1, 2, 4, 8, 16, 32, 64, 128, 256):
         y = gu.bf16_from_dev(h.linear(gu.bf16_to_dev(x[:M])))
         gu.assert_close(y[:, rows], ref[:M], f"{name} {pct}% M={M}")
+        tk = toks_by_m[M]
+        gu.assert_close(y[tk], ref_u[[pos[int(v)] for v in tk]], f"{name} {pct}% M={M}, all rows of tokens {tk.tolist()}")
     sp.check()
 
 

@@ -448,3 +448,16 @@ def test_per_token_activation_quantization_recipe():
         assert abs(int(qx[m, j])) == 127
         assert np.abs(qx[m] * np.float64(sx[m]) - xf[m]).max() <= 0.5 * sx[m] * (1 + 1e-6)
     assert sx[5] == 1 and not qx[5].any()
+
+
+
+def test_layer_sparsity_profile():
+    """The per-layer profile: five levels within +-10 points of 70 %, mean exactly 70 %, as
+    many layers as asked, the same for the same seed."""
+    from paper_2405_03594_gb300 import synth
+
+    for n in (4, 8, 32, 40):
+        p = synth.layer_sparsity_profile(n)
+        assert len(p) == n and sum(p) == 70 * n and set(p) <= {60, 65, 70, 75, 80}
+        assert p == synth.layer_sparsity_profile(n)
+    assert set(synth.layer_sparsity_profile(32)) == {60, 65, 70, 75, 80}
