@@ -63,6 +63,8 @@ def parse():
     ap.add_argument("--no-update", action="store_true", help="skip the masked weight update section")
     ap.add_argument("--square-sweep", action="store_true",
                     help="run only the 12288 x 12288 sparse matmul at 0-90%% sparsity (M = 2048, tensor cores)")
+    ap.add_argument("--no-square", action="store_true", help="skip the 12288 x 12288 sparsity sweep section")
+    ap.add_argument("--no-profile", action="store_true", help="skip the per-layer sparsity profile section")
     ap.add_argument("--no-sweep-config", action="store_true",
                     help="skip the sparsity x batch sweep (gate_up/down, non-uniform masks, M = 1..256)")
     ap.add_argument("--sections-out", default="",
@@ -788,6 +790,10 @@ def run_ours(args):
             sections["masked_update"] = update_section(args, host, peak_gbs)
         if not args.no_sweep_config:
             sections["sparsity_batch_sweep"] = sweep_section(args, peak_gbs)
+        if not args.no_profile:
+            sections["per_layer_profile"] = profile_section(args, peak_gbs)
+        if not args.no_square:
+            sections["square_12288"] = square_section(args)
 
     if rank == 0:
         if args.sections_out:
@@ -823,7 +829,7 @@ def section_summary(sections: dict) -> dict:
     ch = sections.get("chained_step_bf16")
     if ch:
         out["chain_bf16_tok_s"] = {m: _sig(v["tok_s"]) for m, v in ch.get("chain", {}).items()}
-        out["graph_glue_bf16_tok_s"] = {m: _sig(v["tok_s"]) for m, v in ch.get("graph", {}).items()}
+        out["graph_bf16_tok_s"] = {m: _sig(v["tok_s"]) for m, v in ch.get("graph", {}).items()}
     st = sections.get("stack_int8")
     if st:
         out["stack_int8_tok_s"] = {"graph": {m: _sig(v["tok_s"]) for m, v in st.get("graph_per_m", {}).items()},
@@ -841,11 +847,18 @@ def section_summary(sections: dict) -> dict:
         out["vs_dense_cublas"] = {m: _sig(v, 3) for m, v in de["step_speedup"].items()}
     sw = sections.get("sparsity_batch_sweep")
     if sw and sw.get("points"):
-        out["sweep_frac"] = {k: {m: _sig(p["by_m"][m]["frac_of_roofline"], 2) for m in ("1", "16", "64", "256")
+        out["sweep_frac"] = {k: {m: _sig(p["by_m"][m]["frac_of_roofline"], 2) for m in ("16", "256")
                                  if m in p["by_m"]}
                              for k, p in sw["points"].items() if k.endswith("@70%")}
+    pr = sections.get("per_layer_profile")
+    if pr and pr.get("chain"):
+        out["profile_tok_s"] = {"chain": _sig(pr["chain"]["tok_s"]), "graph": _sig(pr.get("graph", {}).get("tok_s"))}
+    sq = sections.get("square_12288")
+    if sq and sq.get("points"):
+        out["square_speedup_vs_0pct"] = {p: _sig(sq["points"][p]["speedup_vs_0pct"], 3) for p in ("50", "70", "90")
+                                         if p in sq["points"]}
     for k in ("chained_step_bf16", "stack_int8", "prefill", "dense_comparison", "masked_update",
-              "sparsity_batch_sweep"):
+              "sparsity_batch_sweep", "per_layer_profile", "square_12288"):
         if sections.get(k) and sections[k].get("error"):
             out.setdefault("errors", {})[k] = str(sections[k]["error"])[:80]
     return out
@@ -927,55 +940,107 @@ def run_single(args):
                       "algorithmic_bytes": nbytes, "gbs": nbytes / (us * 1e-6) / 1e9}), flush=True)
 
 
-def run_square_sweep(args):
-    """The 12288 x 12288 sparse matmul against sparsity (the scaling example of Sec. 2.3 and its
-    12K x 12K figure, measured there on a CS-3; run here on the tensor-core kernel): x [2048, 12288] bf16, per-row magnitude masks at
-    0, 10, ..., 90 %, y = x . (W o M)^T.  Prints one JSON line: per sparsity the launch time,
-    its speedup over the 0 % matrix through the same kernel, the ideal 1 / (1 - s), and the
-    dense cuBLAS GEMM of the same shape for reference.  Opt-in (--square-sweep)."""
+def square_section(args) -> dict:
+    """The 12288 x 12288 sparse matmul against sparsity (the scaling example of Sec. 2.3, there
+    on a CS-3; here on the tensor-core kernel): x [2048, 12288] bf16, per-row magnitude masks at
+    0, 10, ..., 90 %, y = x . (W o M)^T.  Per sparsity the launch time, its speedup over the 0 %
+    matrix through the same kernel, the ideal 1 / (1 - s), and the speedup over the dense cuBLAS
+    GEMM of the same shape.  Parity of this shape is checked by the GPU tests.  A failure is
+    reported in the section instead of ending the run."""
     import torch
 
     from paper_2405_03594_gb300 import sp, synth
 
-    dev = torch.device("cuda", 0)
-    N = K = 12288
-    M = 2048
-    W = synth.weight(N, K, synth.rng(0, 0, 0, synth.STREAM_W))
-    x = synth.activations(M, K, synth.rng(0, 0, 0, synth.STREAM_X))
-    xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
-    y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
-    reps = max(3, min(args.steps, 20))
+    out = {"what": "12288 x 12288, M = 2048, tensor-core kernel, per-row magnitude masks", "N": 12288, "K": 12288,
+           "M": 2048, "kernel": "linear_tc_kernel", "points": {}}
+    try:
+        dev = torch.device("cuda", 0)
+        N = K = 12288
+        M = 2048
+        W = synth.weight(N, K, synth.rng(0, 0, 0, synth.STREAM_W))
+        x = synth.activations(M, K, synth.rng(0, 0, 0, synth.STREAM_X))
+        xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+        y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+        reps = max(3, min(args.steps, 20))
 
-    def timed(fn):
-        for _ in range(3):
-            fn()
-        torch.cuda.synchronize()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record()
-        for _ in range(reps):
-            fn()
-        b.record()
-        torch.cuda.synchronize()
-        return a.elapsed_time(b) / reps * 1e3
+        def timed(fn):
+            for _ in range(3):
+                fn()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(reps):
+                fn()
+            b.record()
+            torch.cuda.synchronize()
+            return a.elapsed_time(b) / reps * 1e3
 
-    Wd = torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16)
-    dense_us = timed(lambda: torch.matmul(xd, Wd.t()))
-    out = {"single": "square_sweep", "N": N, "K": K, "M": M, "kernel": "linear_tc_kernel",
-           "dense_cublas_us": dense_us, "points": {}}
-    base = None
-    for pct in range(0, 100, 10):
-        mask = synth.magnitude_mask(W, pct)
-        h = sp.compress(Wd, torch.from_numpy(mask).to(dev))
-        ws = torch.zeros(max(h.workspace_size(M), 256), dtype=torch.uint8, device=dev)
-        us = timed(lambda: h.linear(xd, out=y, workspace=ws, path="tensor_core"))
-        sp.check()
-        base = us if base is None else base
-        out["points"][str(pct)] = {"us": us, "speedup_vs_0pct": base / us, "ideal": 1.0 / (1.0 - pct / 100.0),
-                                   "speedup_vs_dense_cublas": dense_us / us, "nnz": int(h.info.nnz),
-                                   "compressed_bytes": int(h.info.bytes)}
-        del h, ws
+        Wd = torch.from_numpy(W.view(np.int16)).to(dev).view(torch.bfloat16)
+        dense_us = timed(lambda: torch.matmul(xd, Wd.t()))
+        out["dense_cublas_us"] = dense_us
+        base = None
+        for pct in range(0, 100, 10):
+            mask = synth.magnitude_mask(W, pct)
+            h = sp.compress(Wd, torch.from_numpy(mask).to(dev))
+            ws = torch.zeros(max(h.workspace_size(M), 256), dtype=torch.uint8, device=dev)
+            us = timed(lambda: h.linear(xd, out=y, workspace=ws, path="tensor_core"))
+            sp.check()
+            base = us if base is None else base
+            out["points"][str(pct)] = {"us": us, "speedup_vs_0pct": base / us, "ideal": 1.0 / (1.0 - pct / 100.0),
+                                       "speedup_vs_dense_cublas": dense_us / us, "nnz": int(h.info.nnz),
+                                       "compressed_bytes": int(h.info.bytes)}
+            del h, ws
+            torch.cuda.empty_cache()
+    except Exception as e:  # context only: never let it end the run
+        out["error"] = f"{type(e).__name__}: {e}"
+    return out
+
+
+def run_square_sweep(args):
+    """Only the 12288 x 12288 sweep (--square-sweep): one JSON line."""
+    print(json.dumps({"single": "square_sweep", **square_section(args)}), flush=True)
+
+
+def profile_section(args, peak_gbs) -> dict:
+    """The 32-layer bf16 decode step with a per-layer sparsity profile (60 .. 80 %, mean 70 %;
+    the stand-in for an outlier-weighted layerwise profile): one chained launch per step and a
+    CUDA graph of separate launches, at M = 1, beside the uniform 70 % step of the chained
+    section.  Every layer's masks are drawn at its own sparsity from the seeded layer-0 weights
+    (the five levels' masks, one per shape and level).  Parity of such profiles, linear by
+    linear through both paths, is checked by the GPU tests.  A failure is reported in the
+    section instead of ending the run."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+    from paper_2405_03594_gb300.stack import STACK_WEIGHT_STD, ChainStack, LinearStack
+
+    prof = synth.layer_sparsity_profile(LAYERS)
+    out = {"profile": prof, "mean_pct": sum(prof) / len(prof), "M": 1}
+    try:
+        if not torch.cuda.is_available():
+            raise RuntimeError("no CUDA device")
+        levels = sorted(set(prof))
+        per_level = {p: synth.stack_layer(p, False, seed=0, layer=0, std=STACK_WEIGHT_STD) for p in levels}
+        hosts = [per_level[p] for p in prof]
+        cs = ChainStack(int8=False, max_m=1, host_layers=hosts)
+        ms, cu = time_chain(cs, 1, max(3, min(args.steps, 100)), max(3, args.warmup), 1)
+        b = chain_bytes(cs, 1)
+        out["chain"] = {"tok_s": 1 / (ms * 1e-3), "ms_per_step": ms, "chain_us": cu, "gbs": b / (cu * 1e-6) / 1e9,
+                        "frac_of_peak": b / (cu * 1e-6) / 1e9 / peak_gbs, "weight_bytes": cs.weight_bytes()}
+        del cs
         torch.cuda.empty_cache()
-    print(json.dumps(out), flush=True)
+        st = LinearStack(int8=False, max_m=1, host_layers=hosts)
+        x = synth.activations(1, 4096, synth.rng(0, 0, 0, synth.STREAM_X))
+        st.set_input(torch.from_numpy(x.view(np.int16)).to(st.dev).view(torch.bfloat16))
+        g = st.capture(1)
+        ms = time_graph(g, max(3, min(args.steps, 100)), max(3, args.warmup))
+        sp.check()
+        out["graph"] = {"tok_s": 1 / (ms * 1e-3), "ms_per_step": ms, "launches_per_step": st.launches_per_step(1)}
+        del g, st
+        torch.cuda.empty_cache()
+    except Exception as e:  # context only: never let it end the run
+        out["error"] = f"{type(e).__name__}: {e}"
+    return out
 
 
 def update_bytes(mask: np.ndarray, info) -> int:

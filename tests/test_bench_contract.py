@@ -19,13 +19,13 @@ def _run(*args, timeout=600):
 
 
 def test_reference_arm_prints_one_json_line():
-    p = _run("--impl", "reference", "--steps", "1", "--warmup", "3")
+    p = _run("--impl", "reference", "--steps", "1", "--warmup", "1")
     assert p.returncode == 0, p.stderr[-2000:]
     lines = [ln for ln in p.stdout.splitlines() if ln.strip()]
     assert len(lines) == 1
     d = json.loads(lines[0])
     assert d["impl"] == "reference"
-    assert (d["n_gpus"], d["steps"], d["warmup"]) == (1, 1, 3)
+    assert (d["n_gpus"], d["steps"], d["warmup"]) == (1, 1, 1)
     assert d["unit"] == "tok/s" and d["higher_is_better"] is True and d["vs_baseline"] is None
     assert d["value"] > 0 and d["ms_per_step"] > 0
     M = d["config"]["M"]
@@ -206,6 +206,8 @@ def _full_sections():
         "dense_comparison": {"step_speedup": {"1": 2.3456789, "4": 2.1, "16": 1.9}},
         "sparsity_batch_sweep": {"points": {f"{n}@{p}%": {"by_m": by_m} for n in ("gate_up", "down")
                                             for p in (0, 50, 60, 70, 80)}},
+        "per_layer_profile": {"chain": {"tok_s": 431.12345}, "graph": {"tok_s": 440.12345}},
+        "square_12288": {"points": {str(p): {"speedup_vs_0pct": 1.23456789} for p in range(0, 100, 10)}},
     }
 
 
@@ -238,6 +240,8 @@ def test_headline_line_is_compact_and_complete():
     assert line["config"]["workload"] and line["roofline"]["frac"] == pytest.approx(0.4012, abs=1e-4)
     assert line["value"] == pytest.approx(445.929, rel=1e-5)
     assert set(line["summary"]["sweep_frac"]) == {"gate_up@70%", "down@70%"}
+    assert set(line["summary"]["square_speedup_vs_0pct"]) == {"50", "70", "90"}
+    assert line["summary"]["profile_tok_s"]["chain"] == pytest.approx(431.1, abs=0.1)
     assert "errors" not in line["summary"]
 
 
@@ -245,3 +249,16 @@ def test_section_summary_reports_section_errors():
     b = _bench_module()
     s = b.section_summary({"prefill": {"error": "RuntimeError: " + "x" * 500, "shapes": {}}})
     assert s["errors"]["prefill"].startswith("RuntimeError") and len(s["errors"]["prefill"]) <= 80
+
+
+def test_profile_and_square_sections_report_failures_instead_of_raising():
+    """The per-layer profile and 12K x 12K sections are context: without a GPU they return
+    their failure inside the section rather than ending the run."""
+    import argparse
+
+    b = _bench_module()
+    args = argparse.Namespace(steps=3, warmup=3)
+    pr = b.profile_section(args, 6681.8)
+    assert "error" in pr and sum(pr["profile"]) == 70 * b.LAYERS
+    sq = b.square_section(args)
+    assert "error" in sq and sq["points"] == {}

@@ -294,3 +294,27 @@ def test_shared_workspace_across_grids(sp, oracle):
             y = gu.bf16_from_dev(h.linear(gu.bf16_to_dev(x), workspace=ws))
             gu.assert_close(y, ref, f"rep {rep} N={v.shape[0]}")
     sp.check()
+
+
+@pytest.mark.parametrize("pct", [50, 90])
+def test_square_12288_prefill_parity(sp, oracle, pct):
+    """The 12K x 12K sparse matmul of the sparsity-scaling example (Sec. 2.3), at M = 2048 on
+    the tensor-core kernel as the bench's square sweep runs it: 64 sampled output rows over
+    all tokens (first and last rows included), and every output row for 8 tokens."""
+    import torch
+
+    N = K = 12288
+    W = synth.weight(N, K, synth.rng(0, 0, 0, synth.STREAM_W))
+    mask = synth.magnitude_mask(W, pct)
+    x = synth.activations(2048, K, synth.rng(0, 0, 0, synth.STREAM_X))
+    _, y = _run(sp, W, None, mask, x, path="tensor_core")
+    rows = np.sort(np.random.default_rng(pct).choice(N, 64, replace=False))
+    rows[0], rows[-1] = 0, N - 1
+    ref = oracle.linear_bf16(x, W[rows], mask[rows])
+    got = gu.bf16_from_dev(y[:, torch.from_numpy(rows).to(y.device)])
+    gu.assert_close(got, ref, f"12288^2 {pct}% M=2048, sampled rows")
+    toks = np.concatenate([[0], np.sort(np.random.default_rng(pct + 1).choice(np.arange(1, 2047), 6, replace=False)),
+                           [2047]])
+    ref_t = oracle.linear_bf16(np.ascontiguousarray(x[toks]), W, mask)
+    gu.assert_close(gu.bf16_from_dev(y[torch.from_numpy(toks).to(y.device)]), ref_t,
+                    f"12288^2 {pct}% M=2048, all rows of tokens {toks.tolist()}")
