@@ -105,17 +105,20 @@ sp_status sp_compress(const void* w_dev, const uint8_t* mask_dev, int64_t n, int
                       const float* scale_dev, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx,
                       void* stream, sp_matrix** out);
 
-/* Expand the handle back to the dense masked weight: w_out_dev [N, K] of the
+/* Expand the handle back to the dense masked weight (the inverse of the Sec. 2.4.2 storage:
+ * each submatrix's values placed by its bitmask, Sec. 2.4.1): w_out_dev [N, K] of the
  * handle's dtype (int8 values without their scales for SP_INT8), zero where masked
  * out, bit-exact.  Asynchronous on `stream`; w_out_dev is caller-owned.
  * SP_ERR_BAD_HANDLE for a dead handle, SP_ERR_INVALID_ARG for a null output. */
 sp_status sp_decompress(const sp_matrix* h, void* w_out_dev, void* stream);
 
-/* Bytes of device workspace that sp_linear needs for a batch of m rows, written to
- * *bytes (0 for m == 0).  Host only.  SP_ERR_INVALID_ARG for m < 0 or a null `bytes`. */
+/* Bytes of device workspace that sp_linear needs for a batch of m rows (its split-K scratch;
+ * library plumbing with no counterpart in the paper), written to *bytes (0 for m == 0).  Host only.  SP_ERR_INVALID_ARG for m < 0 or a null `bytes`. */
 sp_status sp_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
 
-/* y = x . (W o Mask)^T, FP32 accumulation, bf16 output (round to nearest even).
+/* y = x . (W o Mask)^T, FP32 accumulation, bf16 output (round to nearest even): the sparse
+ * product of Sec. 2.4.2, the compressed submatrices streamed from global memory and expanded
+ * on chip by their bitmasks; equal to the dense product with the masked weight.
  *   x_dev      [m, K] bf16.      y_dev [m, N] bf16 (fully overwritten).
  *   workspace  device memory of at least sp_workspace_size(h, m) bytes, zero-filled
  *              before its first use; every call leaves it ready for the next one.
@@ -126,7 +129,7 @@ sp_status sp_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
 sp_status sp_linear(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
                     size_t workspace_bytes, void* stream);
 
-/* sp_linear with an explicit kernel family (tests run each family on its own). */
+/* sp_linear (Sec. 2.4.2) with an explicit kernel family (tests run each family on its own). */
 sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
                        size_t workspace_bytes, sp_path path, void* stream);
 
@@ -138,7 +141,8 @@ enum {
   SP_KERNEL_TENSOR_CORE = 3         /* linear_tc_kernel */
 };
 
-/* Number of kernel launches that sp_linear_ex(h, x, m, y, ws, ws_bytes, path, stream)
+/* (Library plumbing; no counterpart in the paper.)  Number of kernel launches that
+ * sp_linear_ex(h, x, m, y, ws, ws_bytes, path, stream)
  * makes, written to *launches: 0 for m == 0, one per 16 batch rows on the CUDA-core
  * family, one on the tensor-core family; if `kernel` is not null, the SP_KERNEL_* value
  * of the kernel used for the first 16 rows (or all rows) goes there.  For callers that
@@ -202,7 +206,8 @@ sp_status sp_masked_update(sp_matrix* h, const float* grad_dev, float lr, void* 
 sp_status sp_linear_w8a8(const sp_matrix* h, const int8_t* qx_dev, const float* sx_dev, int64_t m, void* y_dev,
                          void* workspace_dev, size_t workspace_bytes, void* stream);
 
-/* Workspace bytes sp_linear_w8a8 needs for a batch of m rows (0 for m == 0).  Host only.
+/* Workspace bytes sp_linear_w8a8 (Sec. 3.4) needs for a batch of m rows (0 for m == 0);
+ * library plumbing with no counterpart in the paper.  Host only.
  * SP_ERR_INVALID_ARG for m < 0 or a null `bytes`, SP_ERR_BAD_HANDLE for a dead handle. */
 sp_status sp_w8a8_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
 
@@ -221,31 +226,36 @@ sp_status sp_w8a8_workspace_size(const sp_matrix* h, int64_t m, size_t* bytes);
 sp_status sp_test_expired_wait(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, void* workspace_dev,
                                size_t workspace_bytes, uint32_t wait_ms, void* stream);
 
-/* A copy of the handle with its own device buffers (same bytes), allocated on the
+/* (Library plumbing; no counterpart in the paper.)  A copy of the handle with its own
+ * device buffers (same bytes), allocated on the
  * current device, which must be the handle's (SP_ERR_INVALID_ARG otherwise).  The copies
  * run on `stream`, which is synchronised before the call returns. */
 sp_status sp_clone(const sp_matrix* h, sp_alloc_fn alloc, sp_free_fn free_fn, void* alloc_ctx, void* stream,
                    sp_matrix** out);
 
-/* Release the handle and its device buffers.  The caller must ensure no queued
+/* (Library plumbing; no counterpart in the paper.)  Release the handle and its device
+ * buffers.  The caller must ensure no queued
  * work still reads them (e.g. synchronise the stream first).  NULL is a no-op. */
 sp_status sp_free(sp_matrix* h);
 
-/* Shape and storage facts of a live handle, written to *info (the fields of sp_info_t).
+/* (Library plumbing; no counterpart in the paper.)  Shape and storage facts of a live
+ * handle (the Sec. 2.4.2 storage's sizes), written to *info (the fields of sp_info_t).
  * Host only, no GPU work.  SP_ERR_BAD_HANDLE for a dead handle, SP_ERR_INVALID_ARG for a
  * null `info`. */
 sp_status sp_info(const sp_matrix* h, sp_info_t* info);
 
-/* Synchronously copy the compressed bytes (info.bytes) and the RB*T+1 chunk
+/* (Library plumbing; no counterpart in the paper.)  Synchronously copy the compressed
+ * bytes (info.bytes) and the RB*T+1 chunk
  * offsets (uint64) to host memory; either destination may be NULL. */
 sp_status sp_copy_out(const sp_matrix* h, void* buf_host, size_t buf_cap, uint64_t* off_host, size_t off_count);
 
-/* Synchronise `stream`; report and clear the current device's status word.
+/* (Library plumbing; no counterpart in the paper.)  Synchronise `stream`; report and clear
+ * the current device's status word.
  * Returns SP_ERR_TIMEOUT if a kernel's bounded wait expired since the last
  * check, SP_ERR_CUDA if the stream reported an error, else SP_OK. */
 sp_status sp_check(void* stream);
 
-/* Static English name of a status code. */
+/* Static English name of a status code (library plumbing; no counterpart in the paper). */
 const char* sp_status_string(sp_status s);
 
 #ifdef __cplusplus

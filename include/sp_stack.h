@@ -26,15 +26,19 @@
 extern "C" {
 #endif
 
-/* out[m, j] = in[m, col0 + j] for m < M, j < ncols; in has row stride in_stride elements.
+/* Stack glue (the linear-only stack of the Sec. 3.4 decode measurements, defined above; the
+ * paper defines no such glue): out[m, j] = in[m, col0 + j] for m < M, j < ncols; in has row
+ * stride in_stride elements.
  * ncols, col0 and in_stride must be multiples of 8. */
 sp_status sp_copy_columns(void* out, const void* in, int64_t M, int64_t in_stride, int64_t col0, int64_t ncols,
                           void* stream);
 
-/* h[m, j] = bf16(h[m, j] + a[m, j] + r[j]) in place; h, a [M, N], r [N]; N % 8 == 0. */
+/* Stack glue (as above): h[m, j] = bf16(h[m, j] + a[m, j] + r[j]) in place; h, a [M, N], r [N];
+ * N % 8 == 0. */
 sp_status sp_residual_add(void* h, const void* a, const void* r, int64_t M, int64_t N, void* stream);
 
-/* out[m, j] = bf16(g[m, j] * g[m, F + j]) for j < F; g [M, 2F], out [M, F]; F % 8 == 0. */
+/* Stack glue (as above; the gate * up product of a Llama MLP): out[m, j] = bf16(g[m, j] *
+ * g[m, F + j]) for j < F; g [M, 2F], out [M, F]; F % 8 == 0. */
 sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* stream);
 
 
@@ -66,10 +70,12 @@ typedef struct sp_chain_op {
   int32_t reserved;    /* 0 */
 } sp_chain_op;
 
-/* Workspace bytes that sp_chain_run needs on the current device (0 for m == 0). */
+/* Workspace bytes that sp_chain_run needs on the current device (0 for m == 0); library
+ * plumbing with no counterpart in the paper. */
 sp_status sp_chain_workspace_size(int64_t m, size_t* bytes);
 
-/* Run ops[0], ops[1], ..., ops[n_ops - 1] in order for m batch rows (1 <= m <= 4;
+/* The chained decode step described above (each op a Sec. 2.4.2 sparse linear with its
+ * epilogue).  Run ops[0], ops[1], ..., ops[n_ops - 1] in order for m batch rows (1 <= m <= 4;
  * SP_ERR_UNSUPPORTED above).  All weights live on the current device and hold the same
  * value type (bf16 or INT8).  x, y and r are 2-byte aligned (any row stride); the workspace
  * is 16-byte aligned.  The workspace (sp_chain_workspace_size bytes) is zero-filled before
