@@ -253,15 +253,19 @@ PAPER_SPEEDUPS = {
 def dense_section(host, xs, results, Ms):
     """Context for the paper's sparse-vs-dense speedups: the same layer-0 weights, unpruned,
     as dense bf16 torch.matmul (cuBLAS) launches, timed like the sparse launches (a CUDA
-    graph of back-to-back calls over enough distinct weight copies to exceed 3x L2), and a
-    read-only stream of 1 GiB through a torch reduction.  Not part of the timed step; any
-    failure is reported in the section instead of ending the run."""
+    graph of back-to-back calls over enough distinct weight copies to exceed 3x L2) and as
+    the dense decode step (the 128 launches of 32 layers in layer order, distinct weights per
+    layer, one graph: step_speedup = dense step / sparse step), and a read-only stream of
+    1 GiB through a torch reduction.  Not part of the timed step; any failure is reported in
+    the section instead of ending the run."""
     import numpy as np
     import torch
 
     out = {"how": "dense bf16 torch.matmul (cuBLAS) of the unpruned layer-0 weights, CUDA graph over "
-                  "copies > 3x L2, 20 replays; speedup = dense us / sparse us per launch",
-           "shapes": {}, "step_speedup": {}, "paper": PAPER_SPEEDUPS}
+                  "copies > 3x L2, 20 replays; speedup = dense us / sparse us per launch; step_speedup = "
+                  "dense 32-layer step (128 launches in layer order, 32 weight copies per shape, one graph, "
+                  "10 replays) / the sparse step",
+           "shapes": {}, "step_speedup": {}, "launch_sum_speedup": {}, "paper": PAPER_SPEEDUPS}
     try:
         dev = torch.device("cuda", torch.cuda.current_device())
         dense_sum = {M: 0.0 for M in Ms}
@@ -304,7 +308,38 @@ def dense_section(host, xs, results, Ms):
             out["shapes"][name] = rec
             del ws, w0
             torch.cuda.empty_cache()
-        out["step_speedup"] = {str(M): round(dense_sum[M] / sparse_sum[M], 3) for M in Ms}
+        out["launch_sum_speedup"] = {str(M): round(dense_sum[M] / sparse_sum[M], 3) for M in Ms}
+        # the dense decode step: the same launch sequence as the sparse step
+        layers = [{name: torch.from_numpy(host[name][0].view(np.int16)).to(dev).view(torch.bfloat16)
+                   for name in SHAPES}]
+        layers += [{name: w.clone() for name, w in layers[0].items()} for _ in range(LAYERS - 1)]
+        dense_step = {}
+        for M in Ms:
+            ys = {name: torch.empty((M, layers[0][name].shape[0]), dtype=torch.bfloat16, device=dev)
+                  for name in SHAPES}
+            for name in SHAPES:
+                torch.matmul(xs[name][:M], layers[0][name].t(), out=ys[name])
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                for lw in layers:
+                    for name in SHAPES:
+                        torch.matmul(xs[name][:M], lw[name].t(), out=ys[name])
+            for _ in range(3):
+                g.replay()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for _ in range(10):
+                g.replay()
+            b.record()
+            torch.cuda.synchronize()
+            dense_step[M] = a.elapsed_time(b) / 10
+            del g, ys
+        del layers
+        torch.cuda.empty_cache()
+        out["dense_step_ms"] = {str(M): round(v, 4) for M, v in dense_step.items()}
+        out["step_speedup"] = {str(M): round(dense_step[M] / results[M]["step_ms"], 3) for M in Ms}
         buf = torch.zeros(2 ** 28, dtype=torch.float32, device=dev)
         acc = torch.empty((), dtype=torch.float32, device=dev)
         torch.sum(buf, dim=0, out=acc)

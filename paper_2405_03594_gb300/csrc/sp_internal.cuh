@@ -255,8 +255,9 @@ __device__ __forceinline__ uint16_t float_to_bf16_bits_rn(float f) {
 sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t K, sp_dtype dt, const float* scale,
                           sp_alloc_fn alloc, sp_free_fn free_fn, void* ctx, cudaStream_t stream, sp_matrix** out);
 sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream);
-// allow_cluster: split small row-block counts over thread-block clusters (no workspace
-// needed); otherwise stream-K with split-K partials in the workspace.
+// allow_cluster: each launch takes the split cluster_cc models fastest for its batch rows:
+// a thread-block cluster over each row block (no workspace needed) or stream-K with
+// split-K partials in the workspace; without it every launch is stream-K.
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream, bool allow_cluster = true, uint64_t probe_ns = 0);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);

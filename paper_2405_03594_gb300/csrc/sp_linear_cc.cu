@@ -36,6 +36,12 @@ constexpr int kMaxDevices = 64;
 constexpr int kCtasPerSm = 4;
 constexpr size_t kSmemBudget = 53 * 1024;  // ring slots per CTA; four CTAs share one SM
 constexpr size_t kSmemOptIn = 54 * 1024;
+// Warp-per-chunk cluster launches at M = 1 run six CTAs per SM (64 registers, no spills;
+// 24 consumer warps per SM instead of 16 to cover the walk's latencies) when four ring
+// slots of the matrix's largest chunk fit the smaller budget; other launches spill at 64
+// registers and keep four.
+constexpr int kCtasPerSmM1 = 6;
+constexpr size_t kSmemBudgetM1 = 37 * 1024;
 
 // CTA's work items [w0, w1): a contiguous run of chunks (stream-K), or -- in cluster
 // mode -- K-tiles [r*T/S, (r+1)*T/S) of the row block of its cluster (r = its rank).
@@ -57,10 +63,15 @@ __device__ __forceinline__ void cta_range(const LinearParams& p, bool clustered,
 // x[m, 64t : 64t+64) per batch row into ring slot n % slots, in item order.  The whole
 // warp walks the chunk list (it shares the offset window); lane 0 issues.  Weight bytes
 // do not depend on the previous kernel in the stream: the first ring fill is issued
-// before griddepcontrol.wait; every x copy comes after it.
+// before griddepcontrol.wait; every x copy comes after it.  EARLY: release the next
+// launch in the stream as soon as the dependency is met (the six-CTA M = 1 launches);
+// otherwise the release comes with the CTA's exit.  Measured on GB300 (32-layer decode
+// step, 70%): releasing at exit made the four-CTA launches' steps 6-7% faster at M = 4
+// and 8 (their CTAs no longer land in whatever slots the previous launch's tail leaves),
+// while at M = 1 early release is what lets six-CTA launches overlap.
 // tag[s] = n records that slot s has been claimed for item n (written once the slot's
 // previous item has been consumed), for consumers that do not read every item.
-template <int M>
+template <int M, bool EARLY = true>
 __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, uint64_t* full, uint64_t* empty,
                                         volatile int* tag, int64_t w0, int64_t w1, int lane) {
   const int T = p.T;
@@ -85,7 +96,7 @@ __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, ui
     }
   }
   pdl_wait();
-  pdl_launch_dependents();
+  if constexpr (EARLY) pdl_launch_dependents();
   int s = 0;
   uint32_t ph = 0;
   int t = (int)(w0 % T);
@@ -263,13 +274,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_cc_kernel(const L
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    produce<M>(p, smem, full, empty, tag, w0, w1, lane);
+    produce<M, false>(p, smem, full, empty, tag, w0, w1, lane);
     return;
   }
 
   // -------------------------------------------------------------- consumers
   pdl_wait();  // y, the workspace and x belong to the stream order
-  pdl_launch_dependents();
   float acc[M];
 #pragma unroll
   for (int m = 0; m < M; ++m) acc[m] = 0.f;
@@ -485,8 +495,8 @@ __device__ __forceinline__ void flush_async(const LinearParams& p, FlushCtl* ctl
 // order (deterministic): in stream-K mode by the last warp to get there, which runs the
 // row block's end alone while the others go on (flush_async); in cluster mode, where a
 // CTA's one row block ends with its range, by thread r <-> row r after a barrier.
-template <int M, int ES, bool CL, bool PROBE = false>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const LinearParams p) {
+template <int M, int ES, bool CL, bool PROBE = false, int OCC = kCtasPerSm>
+__global__ void __launch_bounds__(kThreads, OCC) linear_ccw_kernel(const LinearParams p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)p.slots * p.slot_bytes);
@@ -520,12 +530,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    produce<M>(p, smem, full, empty, tag, w0, w1, lane);
+    produce<M, OCC == kCtasPerSmM1>(p, smem, full, empty, tag, w0, w1, lane);
     return;
   }
 
   pdl_wait();
-  pdl_launch_dependents();
+  if constexpr (OCC == kCtasPerSmM1) pdl_launch_dependents();
   bool dead = false;
   if (PROBE && blockIdx.x == 0 && warp == 0) {
     // failure-path test: a bounded wait on a barrier that nothing completes and no copy
@@ -630,10 +640,17 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) linear_ccw_kernel(const 
 
 // kind 0: thread-per-row kernel; kind 1: warp-per-chunk kernel (M <= 4)
 template <int M, int ES>
-sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, bool pdl) {
+sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, int occ, bool pdl) {
   void (*kern)(const LinearParams);
   if constexpr (M <= 4) {
-    if (kind == 1 && p.probe_ns != 0) {
+    if (occ == kCtasPerSmM1) {
+      if constexpr (M == 1) {
+        if (kind != 1 || p.cluster < 2 || p.probe_ns != 0) return SP_ERR_UNSUPPORTED;
+        kern = linear_ccw_kernel<1, ES, true, false, kCtasPerSmM1>;
+      } else {
+        return SP_ERR_UNSUPPORTED;
+      }
+    } else if (kind == 1 && p.probe_ns != 0) {
       if constexpr (ES == 2)
         kern = p.cluster > 1 ? linear_ccw_kernel<M, ES, true, true> : linear_ccw_kernel<M, ES, false, true>;
       else
@@ -645,12 +662,13 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, in
   } else {
     kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
   }
-  static bool configured[3][2][kMaxDevices] = {};  // kernel attributes, once per device
+  static bool configured[4][2][kMaxDevices] = {};  // kernel attributes, once per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
   const int ci = p.cluster > 1 ? 1 : 0;
-  const int ki = p.probe_ns != 0 ? 2 : kind;  // the probe variant is a kernel of its own
+  // the probe variant and the six-CTA variant are kernels of their own
+  const int ki = occ == kCtasPerSmM1 ? 3 : p.probe_ns != 0 ? 2 : kind;
   if (!configured[ki][ci][dev]) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess ||
         (ci && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
@@ -685,44 +703,53 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, in
 }
 
 template <int ES>
-sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, bool pdl) {
+sp_status dispatch_m(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, int occ, bool pdl) {
   switch (p.M) {
-    case 1: return launch_one<1, ES>(p, stream, smem, kind, pdl);
-    case 2: return launch_one<2, ES>(p, stream, smem, kind, pdl);
-    case 3: return launch_one<3, ES>(p, stream, smem, kind, pdl);
-    case 4: return launch_one<4, ES>(p, stream, smem, kind, pdl);
-    case 5: return launch_one<5, ES>(p, stream, smem, kind, pdl);
-    case 6: return launch_one<6, ES>(p, stream, smem, kind, pdl);
-    case 7: return launch_one<7, ES>(p, stream, smem, kind, pdl);
-    case 8: return launch_one<8, ES>(p, stream, smem, kind, pdl);
-    case 9: return launch_one<9, ES>(p, stream, smem, kind, pdl);
-    case 10: return launch_one<10, ES>(p, stream, smem, kind, pdl);
-    case 11: return launch_one<11, ES>(p, stream, smem, kind, pdl);
-    case 12: return launch_one<12, ES>(p, stream, smem, kind, pdl);
-    case 13: return launch_one<13, ES>(p, stream, smem, kind, pdl);
-    case 14: return launch_one<14, ES>(p, stream, smem, kind, pdl);
-    case 15: return launch_one<15, ES>(p, stream, smem, kind, pdl);
-    case 16: return launch_one<16, ES>(p, stream, smem, kind, pdl);
+    case 1: return launch_one<1, ES>(p, stream, smem, kind, occ, pdl);
+    case 2: return launch_one<2, ES>(p, stream, smem, kind, occ, pdl);
+    case 3: return launch_one<3, ES>(p, stream, smem, kind, occ, pdl);
+    case 4: return launch_one<4, ES>(p, stream, smem, kind, occ, pdl);
+    case 5: return launch_one<5, ES>(p, stream, smem, kind, occ, pdl);
+    case 6: return launch_one<6, ES>(p, stream, smem, kind, occ, pdl);
+    case 7: return launch_one<7, ES>(p, stream, smem, kind, occ, pdl);
+    case 8: return launch_one<8, ES>(p, stream, smem, kind, occ, pdl);
+    case 9: return launch_one<9, ES>(p, stream, smem, kind, occ, pdl);
+    case 10: return launch_one<10, ES>(p, stream, smem, kind, occ, pdl);
+    case 11: return launch_one<11, ES>(p, stream, smem, kind, occ, pdl);
+    case 12: return launch_one<12, ES>(p, stream, smem, kind, occ, pdl);
+    case 13: return launch_one<13, ES>(p, stream, smem, kind, occ, pdl);
+    case 14: return launch_one<14, ES>(p, stream, smem, kind, occ, pdl);
+    case 15: return launch_one<15, ES>(p, stream, smem, kind, occ, pdl);
+    case 16: return launch_one<16, ES>(p, stream, smem, kind, occ, pdl);
     default: return SP_ERR_INVALID_ARG;
   }
 }
 
-// Thread-block cluster split: each row block is split over S CTAs of one cluster
-// (S <= 16, S <= T, all CTAs within kCtasPerSm per SM), which replaces the global
-// split-K fix-up by a distributed-shared-memory reduction.  Taken when the clusters fill
-// at least 80% of the CTA slots (measured: on the 172 row blocks of gate/up, 3-CTA
-// clusters filling 85% beat stream-K over all slots), or when the matrix is small (few
-// row blocks: there the fixed latency of the global fix-up dominates); otherwise stream-K
-// balances better.
-int cluster_cc(const sp_matrix* h) {
-  const int64_t cap = (int64_t)kCtasPerSm * h->num_sms;
+// Thread-block cluster split: each row block is split over S CTAs of one cluster, which
+// replaces the global split-K fix-up by a distributed-shared-memory reduction; S = 1 is the
+// stream-K launch over grid_cc CTAs, taken only when not even two CTAs per row block fit
+// the SMs' CTA slots.  S is the largest cluster size that fits the slots (occ CTAs per
+// SM) and leaves each CTA at least cmin chunks (at least two ranks when the row block is
+// short), from 2..8 and 16.  Measured on GB300 (decode steps of the 32-layer Llama-2-7B
+// stack, 70%, bf16 and INT8): a step ran fastest when every launch's grid filled most of
+// the slots, because each launch then overlaps evenly with its neighbours under
+// programmatic dependent launch; small grids that won alone (q/k/v in 288 CTAs instead
+// of 576) cost up to 6 us per layer in the step.  With four CTAs per SM, 4-chunk CTAs (o,
+// S = 16) lost to 8-chunk ones (cmin = 8); with six they won (cmin = 4).  Cluster sizes
+// 9..15 ran 35% slower than 8 on down and are not taken.  Choices: four CTAs per SM --
+// q/k/v (96 row blocks) 6, o (32) 8, gate/up (172) 3, down (32 of 172 chunks) 16; six --
+// 8, 16, 5, 16.
+int cluster_cc(const sp_matrix* h, int occ) {
   const int64_t rb = std::max<int32_t>(h->RB, 1);
-  int64_t S = std::min<int64_t>(16, cap / rb);
-  S = std::min<int64_t>(S, h->T);
-  if (S < 2) return 1;
-  const bool fills = 10 * rb * S >= 8 * cap;
-  const bool small = 8 * rb <= cap;
-  return (fills || small) ? (int)S : 1;
+  const int64_t T = h->T;
+  const int64_t smax = std::min<int64_t>(std::min<int64_t>(16, (int64_t)occ * h->num_sms / rb), T);
+  if (smax < 2) return 1;
+  const int64_t cmin = std::min<int64_t>(occ == kCtasPerSm ? 8 : 4, (T + 1) / 2);
+  for (int64_t S = smax; S > 2; --S) {
+    if (S > 8 && S < 16) continue;
+    if ((T + S - 1) / S >= cmin) return (int)S;
+  }
+  return 2;
 }
 
 int grid_cc(const sp_matrix* h) {
@@ -737,11 +764,11 @@ int grid_cc(const sp_matrix* h) {
 // warp-per-chunk kernel runs (M <= 4 and room for a slot per consumer warp after its
 // partials), and the offsets of the warps' partials and of the cluster partial.
 struct CcPlan {
-  int slots, kind;
+  int slots, kind, occ;
   uint32_t slot_bytes, comb_off, part_off;
   size_t smem;
 };
-bool cc_plan(const sp_matrix* h, int Mt, int S, CcPlan* pl) {
+bool cc_plan(const sp_matrix* h, int Mt, int S, int occ, CcPlan* pl) {
   const uint32_t chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
   pl->slot_bytes = chunk_region + (uint32_t)Mt * 128u;
   // shared memory: ring slots, 2*slots mbarriers (<= 256 B), the flag (16 B), the slot
@@ -750,13 +777,14 @@ bool cc_plan(const sp_matrix* h, int Mt, int S, CcPlan* pl) {
   const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
   const size_t comb_bytes = 2 * (size_t)kConsumerWarps * kRows * Mt * sizeof(float) + sizeof(FlushCtl);
   pl->kind = 0;
-  size_t ring = kSmemBudget - 256 - 16 - 64 - part_bytes;
+  pl->occ = occ;
+  size_t ring = (occ == kCtasPerSmM1 ? kSmemBudgetM1 : kSmemBudget) - 256 - 16 - 64 - part_bytes;
   if (Mt <= 4 && (ring - comb_bytes) / pl->slot_bytes >= (size_t)kConsumerWarps) {
     pl->kind = 1;
     ring -= comb_bytes;
   }
   pl->slots = (int)std::min<size_t>(16, ring / pl->slot_bytes);
-  if (pl->slots < 2) return false;
+  if (pl->slots < 2 || (occ == kCtasPerSmM1 && pl->kind != 1)) return false;
   pl->comb_off = (uint32_t)(((size_t)pl->slots * pl->slot_bytes + 2 * (size_t)pl->slots * 8 + 16 +
                              4 * (size_t)pl->slots + 15) /
                             16 * 16);
@@ -765,11 +793,27 @@ bool cc_plan(const sp_matrix* h, int Mt, int S, CcPlan* pl) {
   return true;
 }
 
+// The launch configuration of one launch with Mt batch rows: six CTAs per SM for a
+// warp-per-chunk cluster launch at M = 1 where its plan fits, else four; S = 1 (stream-K)
+// without clusters.
+bool select_cc(const sp_matrix* h, int Mt, bool allow_cluster, bool probe, int* S, CcPlan* pl) {
+  if (allow_cluster && Mt == 1 && !probe) {
+    const int s1 = cluster_cc(h, kCtasPerSmM1);
+    if (s1 > 1 && cc_plan(h, 1, s1, kCtasPerSmM1, pl)) {
+      *S = s1;
+      return true;
+    }
+  }
+  *S = allow_cluster ? cluster_cc(h, kCtasPerSm) : 1;
+  return cc_plan(h, Mt, *S, kCtasPerSm, pl);
+}
+
 }  // namespace
 
 int cc_kernel_kind(const sp_matrix* h, int64_t M) {
   CcPlan pl;
-  return cc_plan(h, (int)std::min<int64_t>(kMaxTokens, M), cluster_cc(h), &pl) ? pl.kind : -1;
+  int S;
+  return select_cc(h, (int)std::min<int64_t>(kMaxTokens, M), true, false, &S, &pl) ? pl.kind : -1;
 }
 
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
@@ -779,9 +823,18 @@ size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
 
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream, bool allow_cluster, uint64_t probe_ns) {
-  const int S = allow_cluster ? cluster_cc(h) : 1;
+  // the configuration depends on the batch rows of a launch: full launches of kMaxTokens
+  // rows and one ragged tail; the workspace is checked before the first launch
+  const bool probe = probe_ns != 0;
+  auto stream_k = [&](int Mt) {
+    CcPlan q;
+    int S = 1;
+    return !select_cc(h, Mt, allow_cluster, probe, &S, &q) || S == 1;
+  };
+  const int tail = (int)(M % kMaxTokens);
+  const bool needs_ws = (M >= kMaxTokens && stream_k(kMaxTokens)) || (tail != 0 && stream_k(tail));
   const size_t need = workspace_bytes_cc(h, M);
-  if (S == 1 && (!ws || ws_bytes < need)) return SP_ERR_WORKSPACE;
+  if (needs_ws && (!ws || ws_bytes < need)) return SP_ERR_WORKSPACE;
   LinearParams p{};
   p.buf = h->d_buf;
   p.off = h->d_off;
@@ -792,8 +845,6 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.T = h->T;
   p.RB = h->RB;
   p.W = (int64_t)h->RB * h->T;
-  p.cluster = S;
-  p.G = S > 1 ? h->RB * S : grid_cc(h);
   p.cnt = reinterpret_cast<int*>(ws);
   p.ws = ws ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms)) : nullptr;
   p.timeout_ns = wait_timeout_ns();
@@ -801,11 +852,14 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
   for (int64_t m0 = 0; m0 < M; m0 += kMaxTokens) {
     const int Mt = (int)std::min<int64_t>(kMaxTokens, M - m0);
+    int S = 1;
+    CcPlan pl;
+    if (!select_cc(h, Mt, allow_cluster, probe, &S, &pl)) return SP_ERR_UNSUPPORTED;
     p.M = Mt;
+    p.cluster = S;
+    p.G = S > 1 ? h->RB * S : grid_cc(h);
     p.x = x + m0 * h->K;
     p.y = y + m0 * h->N;
-    CcPlan pl;
-    if (!cc_plan(h, Mt, S, &pl)) return SP_ERR_UNSUPPORTED;
     p.slot_bytes = pl.slot_bytes;
     p.slots = pl.slots;
     p.comb_off = pl.comb_off;
@@ -815,8 +869,8 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     // after an in-place weight update the first launch waits for the whole previous grid
     // (no weight copy may start before its writes are visible)
     const bool pdl = !(m0 == 0 && h->weights_written);
-    const sp_status st =
-        h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind, pdl) : dispatch_m<1>(p, stream, smem, kind, pdl);
+    const sp_status st = h->esize == 2 ? dispatch_m<2>(p, stream, smem, kind, pl.occ, pdl)
+                                        : dispatch_m<1>(p, stream, smem, kind, pl.occ, pdl);
     if (st != SP_OK) return st;
     h->weights_written = 0;
   }

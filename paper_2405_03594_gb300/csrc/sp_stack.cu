@@ -1,5 +1,15 @@
 // sp_stack.cu -- elementwise glue of the linear-stack decode step (include/sp_stack.h).
 // Each thread moves 8 bf16 (16 bytes) per access; FP32 arithmetic, one RNE rounding.
+// Launched with programmatic dependent launch, like the sparse linears around them: a
+// kernel's CTAs become resident while the previous grid runs and read nothing before
+// griddepcontrol.wait (which returns once every earlier grid of the stream has completed).
+// At M = 1 a glue kernel releases the next launch at once, so the next linear's CTAs
+// become resident and copy weights while the glue runs; at M > 1 the release comes with
+// the glue's exit.  Measured on GB300 (graph of the 32-layer step, 70%): early release
+// 450 / 1277 tok/s at M = 1 / 4 (bf16), release at exit 432 / 1358, no PDL 446 / 1144;
+// the M = 1 linears run six CTAs per SM and gain from early residency, the four-per-SM
+// M > 1 linears lose by it (their CTAs land unevenly in the slots the previous linear's
+// tail leaves).
 #include "../../include/sp_stack.h"
 #include "sp_internal.cuh"
 
@@ -14,8 +24,14 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
   return (uint32_t)float_to_bf16_bits_rn(a) | ((uint32_t)float_to_bf16_bits_rn(b) << 16);
 }
 
+__device__ __forceinline__ void glue_begin(bool early_release) {
+  pdl_wait();
+  if (early_release) pdl_launch_dependents();
+}
+
 __global__ void copy_columns_kernel(uint4* __restrict__ out, const uint4* __restrict__ in, int64_t M,
-                                    int64_t in_stride8, int64_t col8, int64_t ncols8) {
+                                    int64_t in_stride8, int64_t col8, int64_t ncols8, bool early_release) {
+  glue_begin(early_release);
   const int64_t total = M * ncols8;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t m = i / ncols8, j = i % ncols8;
@@ -24,7 +40,8 @@ __global__ void copy_columns_kernel(uint4* __restrict__ out, const uint4* __rest
 }
 
 __global__ void residual_add_kernel(uint4* __restrict__ h, const uint4* __restrict__ a, const uint4* __restrict__ r,
-                                    int64_t M, int64_t n8) {
+                                    int64_t M, int64_t n8, bool early_release) {
+  glue_begin(early_release);
   const int64_t total = M * n8;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const uint4 hv = h[i], av = a[i], rv = r[i % n8];
@@ -37,7 +54,9 @@ __global__ void residual_add_kernel(uint4* __restrict__ h, const uint4* __restri
   }
 }
 
-__global__ void mul_halves_kernel(uint4* __restrict__ out, const uint4* __restrict__ g, int64_t M, int64_t f8) {
+__global__ void mul_halves_kernel(uint4* __restrict__ out, const uint4* __restrict__ g, int64_t M, int64_t f8,
+                                  bool early_release) {
+  glue_begin(early_release);
   const int64_t total = M * f8;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t m = i / f8, j = i % f8;
@@ -53,11 +72,23 @@ __global__ void mul_halves_kernel(uint4* __restrict__ out, const uint4* __restri
 
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-unsigned grid_for(int64_t total) {
+template <typename... Params, typename... Args>
+sp_status launch_glue(void (*kern)(Params...), int64_t total, cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
   int64_t b = (total + kBlock - 1) / kBlock;
-  if (b < 1) b = 1;
-  if (b > 4096) b = 4096;
-  return (unsigned)b;
+  cfg.gridDim = dim3((unsigned)(b < 1 ? 1 : b > 4096 ? 4096 : b));
+  cfg.blockDim = dim3(kBlock);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, kern, args...) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
+  return SP_OK;
 }
 
 }  // namespace
@@ -73,9 +104,8 @@ sp_status sp_copy_columns(void* out, const void* in, int64_t M, int64_t in_strid
   if (ncols % 8 || col0 % 8 || in_stride % 8) return SP_ERR_UNSUPPORTED;
   if (!al16(out) || !al16(in)) return SP_ERR_ALIGNMENT;
   if (M == 0 || ncols == 0) return SP_OK;
-  copy_columns_kernel<<<grid_for(M * ncols / 8), kBlock, 0, (cudaStream_t)stream>>>(
-      (uint4*)out, (const uint4*)in, M, in_stride / 8, col0 / 8, ncols / 8);
-  return cudaGetLastError() == cudaSuccess ? SP_OK : SP_ERR_CUDA;
+  return launch_glue(copy_columns_kernel, M * ncols / 8, (cudaStream_t)stream, (uint4*)out, (const uint4*)in, M,
+                     in_stride / 8, col0 / 8, ncols / 8, M == 1);
 }
 
 sp_status sp_residual_add(void* h, const void* a, const void* r, int64_t M, int64_t N, void* stream) {
@@ -83,9 +113,8 @@ sp_status sp_residual_add(void* h, const void* a, const void* r, int64_t M, int6
   if (N % 8) return SP_ERR_UNSUPPORTED;
   if (!al16(h) || !al16(a) || !al16(r)) return SP_ERR_ALIGNMENT;
   if (M == 0 || N == 0) return SP_OK;
-  residual_add_kernel<<<grid_for(M * N / 8), kBlock, 0, (cudaStream_t)stream>>>((uint4*)h, (const uint4*)a,
-                                                                                (const uint4*)r, M, N / 8);
-  return cudaGetLastError() == cudaSuccess ? SP_OK : SP_ERR_CUDA;
+  return launch_glue(residual_add_kernel, M * N / 8, (cudaStream_t)stream, (uint4*)h, (const uint4*)a,
+                     (const uint4*)r, M, N / 8, M == 1);
 }
 
 sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* stream) {
@@ -93,8 +122,8 @@ sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* st
   if (F % 8) return SP_ERR_UNSUPPORTED;
   if (!al16(out) || !al16(g)) return SP_ERR_ALIGNMENT;
   if (M == 0 || F == 0) return SP_OK;
-  mul_halves_kernel<<<grid_for(M * F / 8), kBlock, 0, (cudaStream_t)stream>>>((uint4*)out, (const uint4*)g, M, F / 8);
-  return cudaGetLastError() == cudaSuccess ? SP_OK : SP_ERR_CUDA;
+  return launch_glue(mul_halves_kernel, M * F / 8, (cudaStream_t)stream, (uint4*)out, (const uint4*)g, M, F / 8,
+                     M == 1);
 }
 
 }  // extern "C"
