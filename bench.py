@@ -61,6 +61,7 @@ def parse():
     ap.add_argument("--no-prefill", action="store_true", help="skip the M=2048 prefill section")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense cuBLAS comparison section")
     ap.add_argument("--no-update", action="store_true", help="skip the masked weight update section")
+    ap.add_argument("--no-w8a8", action="store_true", help="skip the INT8-activation (W8A8) section")
     ap.add_argument("--square-sweep", action="store_true",
                     help="run only the 12288 x 12288 sparse matmul at 0-90%% sparsity (M = 2048, tensor cores)")
     ap.add_argument("--no-square", action="store_true", help="skip the 12288 x 12288 sparsity sweep section")
@@ -823,6 +824,8 @@ def run_ours(args):
             sections["dense_comparison"] = dense_section(host, xs, results, Ms)
         if not args.no_update:
             sections["masked_update"] = update_section(args, host, peak_gbs)
+        if not args.no_w8a8:
+            sections["w8a8"] = w8a8_section(args, host, peak_gbs)
         if not args.no_sweep_config:
             sections["sparsity_batch_sweep"] = sweep_section(args, peak_gbs)
         if not args.no_profile:
@@ -872,11 +875,15 @@ def section_summary(sections: dict) -> dict:
     pf = sections.get("prefill")
     if pf and pf.get("shapes"):
         fr = {k: v["frac_dense_executed"] for k, v in pf["shapes"].items()}
-        out["prefill_frac_dense"] = {"min": _sig(min(fr.values()), 3), "max": _sig(max(fr.values()), 3),
-                                     "qkv@70%": _sig(fr.get("qkv@70%"), 3)}
+        out["prefill_frac_dense"] = {"min": _sig(min(fr.values()), 3), "max": _sig(max(fr.values()), 3)}
     up = sections.get("masked_update")
     if up and up.get("shapes"):
         out["update_frac"] = {n: _sig(v["frac"], 3) for n, v in up["shapes"].items()}
+    wa = sections.get("w8a8")
+    if wa and wa.get("shapes", {}).get("gate_up"):
+        # gate_up: time of sp_linear_w8a8 / time of the INT8-weight linear on bf16 x
+        out["w8a8_rel"] = {m: _sig(v["w8a8_over_int8_weight"], 3) for m, v in wa["shapes"]["gate_up"].items()
+                           if m in ("1", "64")}
     de = sections.get("dense_comparison")
     if de and de.get("step_speedup"):
         out["vs_dense_cublas"] = {m: _sig(v, 3) for m, v in de["step_speedup"].items()}
@@ -892,7 +899,7 @@ def section_summary(sections: dict) -> dict:
     if sq and sq.get("points"):
         out["square_speedup_vs_0pct"] = {p: _sig(sq["points"][p]["speedup_vs_0pct"], 3) for p in ("50", "70", "90")
                                          if p in sq["points"]}
-    for k in ("chained_step_bf16", "stack_int8", "prefill", "dense_comparison", "masked_update",
+    for k in ("chained_step_bf16", "stack_int8", "prefill", "dense_comparison", "masked_update", "w8a8",
               "sparsity_batch_sweep", "per_layer_profile", "square_12288"):
         if sections.get(k) and sections[k].get("error"):
             out.setdefault("errors", {})[k] = str(sections[k]["error"])[:80]
@@ -1164,6 +1171,69 @@ def sweep_section(args, peak_gbs):
     except Exception as e:  # context only: never let it end the run
         res["error"] = f"{type(e).__name__}: {e}"
     torch.cuda.empty_cache()
+    return res
+
+
+def w8a8_section(args, host, peak_gbs):
+    """INT8 weights with INT8 activations (sp_linear_w8a8: per-token absmax x, widened to bf16
+    by one launch, then the INT8-weight linear) against the INT8-weight linear alone on bf16
+    x, gate_up and down at the bench's sparsity, M = 1 / 16 / 64; back-to-back calls over
+    enough distinct copies of the compressed matrix to exceed 3x L2.  Context next to the
+    decode step; a failure is reported in the section and never ends the run."""
+    import torch
+
+    from paper_2405_03594_gb300 import sp, synth
+
+    dev = torch.device("cuda", 0)
+    res = {"what": "sp_linear_w8a8 (2 launches) vs sp_linear on INT8 weights with bf16 x", "shapes": {}}
+    try:
+        for name in ("gate_up", "down"):
+            W, mask, _ = host[name]
+            q, sc = synth.quantize_int8(W, mask)
+            h0 = sp.compress(torch.from_numpy(q).to(dev), torch.from_numpy(mask).to(dev),
+                             torch.from_numpy(sc).to(dev))
+            copies = max(2, int(-(-3 * L2_BYTES // int(h0.info.bytes))))
+            hs = [h0] + [h0.clone() for _ in range(copies - 1)]
+            rec = {}
+            for M in (1, 16, 64):
+                x = synth.activations(M, h0.k, synth.rng(0, 0, 7, synth.STREAM_X))
+                qx, sx = synth.quantize_activations_int8(x)
+                qxd, sxd = torch.from_numpy(qx).to(dev), torch.from_numpy(sx).to(dev)
+                xd = torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+                y = torch.empty((M, h0.n), dtype=torch.bfloat16, device=dev)
+                ws = torch.zeros(max(h0.w8a8_workspace_size(M), h0.workspace_size(M), 256), dtype=torch.uint8,
+                                 device=dev)
+
+                def timed(fn):
+                    for h in hs:
+                        fn(h)
+                    torch.cuda.synchronize()
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    reps = 10
+                    a.record()
+                    for _ in range(reps):
+                        for h in hs:
+                            fn(h)
+                    b.record()
+                    torch.cuda.synchronize()
+                    sp.check()
+                    return a.elapsed_time(b) / (reps * len(hs)) * 1e3
+
+                us_w8a8 = timed(lambda h: h.linear_w8a8(qxd, sxd, out=y, workspace=ws))
+                us_w8 = timed(lambda h: h.linear(xd, out=y, workspace=ws))
+                nbytes = (int(h0.info.nnz) + h0.n * h0.k // 8 + int(h0.info.scale_bytes) + M * h0.k + 4 * M
+                          + 2 * M * h0.n)
+                rec[str(M)] = {"w8a8_us": round(us_w8a8, 3), "int8_weight_us": round(us_w8, 3),
+                               "w8a8_over_int8_weight": round(us_w8a8 / us_w8, 3),
+                               "w8a8_gbs": round(nbytes / (us_w8a8 * 1e-6) / 1e9, 1),
+                               "w8a8_frac": round(nbytes / (us_w8a8 * 1e-6) / 1e9 / peak_gbs, 3),
+                               "launches": 2}
+                del y, ws
+            res["shapes"][name] = rec
+            del hs, h0
+            torch.cuda.empty_cache()
+    except Exception as e:  # context only: never let it end the run
+        res["error"] = f"{type(e).__name__}: {e}"[:300]
     return res
 
 

@@ -7,7 +7,11 @@
 // once, x[m, k] = bf16_rne(qx[m, k] * sx[m]) (float32 product, one rounding), into the
 // caller's workspace, and runs the INT8-weight sparse linear on that x (its epilogue
 // applies sw[n]).  The widening is one elementwise pass over M x K bytes; every kernel
-// choice of sp_linear (CUDA-core decode, tensor-core prefill) applies unchanged.
+// choice of sp_linear (CUDA-core decode, tensor-core prefill) applies unchanged.  The
+// widening runs under programmatic dependent launch like the linears: it writes x only after
+// griddepcontrol.wait (every earlier grid of the stream has completed), and it releases the
+// linear that follows at once for one-row batches (whose six-CTA launch then copies its
+// weights while the widening runs) and at its exit otherwise, as the stack's glue kernels do.
 #include <algorithm>
 
 #include "sp_internal.cuh"
@@ -20,7 +24,10 @@ constexpr int kWidenBlock = 256;
 // Eight activations per thread: one 8-byte load of qx, one 16-byte store of bf16.
 // K % 8 == 0 (checked at compression), so a row holds K / 8 whole groups.
 __global__ void __launch_bounds__(kWidenBlock) widen_kernel(const uint2* __restrict__ qx, const float* __restrict__ sx,
-                                                            uint4* __restrict__ x, int64_t M, int64_t k8) {
+                                                            uint4* __restrict__ x, int64_t M, int64_t k8,
+                                                            bool early_release) {
+  pdl_wait();
+  if (early_release) pdl_launch_dependents();
   const int64_t total = M * k8;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const float s = sx[i / k8];
@@ -88,8 +95,19 @@ extern "C" sp_status sp_linear_w8a8(const sp_matrix* h, const int8_t* qx_dev, co
   const int64_t total = m * k8;
   const int64_t blocks = std::max<int64_t>(
       1, std::min<int64_t>((total + kWidenBlock - 1) / kWidenBlock, (int64_t)h->num_sms * 8));
-  widen_kernel<<<(unsigned)blocks, kWidenBlock, 0, (cudaStream_t)stream>>>(reinterpret_cast<const uint2*>(qx_dev),
-                                                                         sx_dev, x, m, k8);
-  if (cudaGetLastError() != cudaSuccess) return SP_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(kWidenBlock);
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, widen_kernel, reinterpret_cast<const uint2*>(qx_dev), sx_dev, x, m, k8, m == 1) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
   return sp_linear(h, x, m, y_dev, ws, round256(lin), stream);
 }

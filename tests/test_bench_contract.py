@@ -203,6 +203,8 @@ def _full_sections():
                        "chain_per_m": {"1": {"tok_s": 368.12}, "4": {"tok_s": 1048.4}}},
         "prefill": {"shapes": {f"{n}@{p}%": {"frac_dense_executed": 0.3212345} for n in per_shape for p in (50, 70)}},
         "masked_update": {"shapes": {n: {"frac": 0.4612345} for n in per_shape}},
+        "w8a8": {"shapes": {n: {str(m): {"w8a8_over_int8_weight": 1.2345678} for m in (1, 16, 64)}
+                            for n in ("gate_up", "down")}},
         "dense_comparison": {"step_speedup": {"1": 2.3456789, "4": 2.1, "16": 1.9}},
         "sparsity_batch_sweep": {"points": {f"{n}@{p}%": {"by_m": by_m} for n in ("gate_up", "down")
                                             for p in (0, 50, 60, 70, 80)}},
