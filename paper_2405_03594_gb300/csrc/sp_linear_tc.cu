@@ -17,7 +17,7 @@
 //   warp 1          TMEM allocation; lane 0 issues the MMAs (4 x K=16 per chunk) and
 //                   commits them to mbarriers that free the stage and, at a segment's
 //                   end, hand D to the epilogue;
-//   warps 2-9       two expander warpgroups taking alternate chunks: thread r of a
+//   warps 2-..      EG expander warpgroups taking chunks round-robin: thread r of a
 //                   warpgroup owns TMEM lane / chunk row r; it finds its first value by a
 //                   popc prefix sum, expands 64 columns into 32 bf16x2 registers, and
 //                   stores them to an A stage with tcgen05.st; at a row-block end the
@@ -36,8 +36,16 @@
 namespace sp {
 namespace {
 
-constexpr int kExpGroups = 2;         // expander warpgroups, taking alternate chunks
-constexpr int kThreads = (2 + 4 * kExpGroups) * 32;
+// Expander warpgroups EG (a template parameter: 2 or 3) take items round-robin; a CTA
+// runs 2 + 4 * EG warps.  Three groups (14 warps: three expander warps on each SM
+// sub-partition, at most 128 registers) for token tiles of up to 64 tokens, where the
+// ring still holds two slots per group: at M = 16 the kernel with two groups issued on
+// 42 % of cycles, stalled on fixed-latency and shared-memory results with 10 warps per
+// SM (ncu).  Two groups for wider tiles (their x tiles leave room for few slots).  Four
+// groups (18 warps) would put five warps on two sub-partitions, whose 16K registers then
+// allow 96 per thread: ~300 bytes of spills.
+constexpr int kMaxExpGroups = 3;
+__host__ __device__ constexpr int tc_threads(int eg) { return (2 + 4 * eg) * 32; }
 constexpr int kExpWarp0 = 2;          // first expander warp
 constexpr int kMaxAStages = 16;       // A tiles in TMEM (32 columns each), at most
 constexpr int kMaxDBufs = 2;          // D accumulators in TMEM (ntok columns each), at most
@@ -219,7 +227,7 @@ struct TcParams {
   uint32_t d_cols;    // TMEM columns per D buffer (ntok rounded up to 32)
   uint32_t a_col0;    // first TMEM column of the A stages (n_d * d_cols)
   int32_t y_tma;      // 1: y is written by TMA stores from a staging tile (needs N % 8 == 0)
-  uint32_t stg_off;   // shared-memory offset of the staging tiles [kExpGroups][2][32][128] bf16
+  uint32_t stg_off;   // shared-memory offset of the staging tiles [EG][2][32][128] bf16
 };
 
 constexpr int kStgTokens = 32;                          // tokens per staged block
@@ -272,22 +280,22 @@ __host__ __device__ inline void tmem_split(int ntok, int* n_a, int* n_d, uint32_
   *d_cols = dc;
 }
 
-template <int ES>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int ES, int EG>
+__global__ void __launch_bounds__(tc_threads(EG), 1)
     linear_tc_kernel(const __grid_constant__ TcParams tp, const __grid_constant__ CUtensorMap tmap_x,
                      const __grid_constant__ CUtensorMap tmap_y) {
   extern __shared__ uint8_t smem_raw[];
   const LinearParams& p = tp.p;
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const int slots = p.slots;
-  // Ring: item n uses slot n % S and A stage n % S (S = slots <= A stages, even).
+  // Ring: item n uses slot n % S and A stage n % S (S = slots <= A stages, a multiple of EG).
   //   full[s]       chunk and x tile landed (producer's expect_tx + the copies)
   //   a_full[s]     the four warps of the item's expander warpgroup stored the A stage
   //   stage_free[s] the item's MMAs completed (one commit): slot and A stage are free.
   // The expanders read the chunk before arriving on a_full, and the MMAs are issued only
   // after a_full, so that one commit also covers the expanders' reads of the slot.  An
   // expander waits only on full[s]: the producer refills a slot only after stage_free,
-  // and with S even a slot's previous item belongs to the same warpgroup.
+  // and with S a multiple of EG a slot's previous item belongs to the same warpgroup.
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)slots * p.slot_bytes);
   uint64_t* stage_free = full + slots;
   uint64_t* a_full = stage_free + slots;
@@ -299,8 +307,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // has finished the previous segment on that buffer).  d_empty has one barrier per
   // buffer: the MMA issuer starts segment k only after the epilogue of segment k - n_d
   // has read that buffer, so those epilogues complete in order.
-  uint64_t* d_full = a_full + slots;                      // [kMaxDBufs][kExpGroups]
-  uint64_t* d_empty = d_full + kMaxDBufs * kExpGroups;    // [kMaxDBufs]
+  uint64_t* d_full = a_full + slots;                      // [kMaxDBufs][EG]
+  uint64_t* d_empty = d_full + kMaxDBufs * kMaxExpGroups; // [kMaxDBufs]
   uint32_t* tmem_base_slot = reinterpret_cast<uint32_t*>(d_empty + kMaxDBufs);
   volatile int* s_flag = reinterpret_cast<volatile int*>(tmem_base_slot + 1);  // one per warpgroup
 
@@ -316,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&stage_free[s], 1);  // one MMA commit
       mbar_init(&a_full[s], 4);      // the four warps of an expander warpgroup
     }
-    for (int b = 0; b < kMaxDBufs * kExpGroups; ++b) mbar_init(&d_full[b], 1);
+    for (int b = 0; b < kMaxDBufs * EG; ++b) mbar_init(&d_full[b], 1);
     for (int b = 0; b < kMaxDBufs; ++b) mbar_init(&d_empty[b], 4);  // the epilogue warpgroup's four warps
     fence_barrier_init();
   }
@@ -437,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_ts(d_taddr, a_taddr + (uint32_t)kk * 8u, bdesc, idesc, (seg_first && kk == 0) ? 0u : 1u);
           }
           mma_commit(&stage_free[s]);
-          if (seg_last) mma_commit(&d_full[db * kExpGroups + (int)((w - w0) % kExpGroups)]);
+          if (seg_last) mma_commit(&d_full[db * EG + (int)((w - w0) % EG)]);
         }
         if (++s == slots) {
           s = 0;
@@ -456,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tid128 = (warp - kExpWarp0 - 4 * grp) * 32 + lane;
     bool dead = false;
     const int64_t sg_first = w0 / T;
-    // ring position of item n = grp, grp + kExpGroups, ... (slots >= kExpGroups)
+    // ring position of item n = grp, grp + EG, ... (slots a multiple of EG)
     int s = grp;
     uint32_t ph = 0;
     int t = (int)((w0 + grp) % T);  // K-tile of item w
@@ -464,9 +472,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint16_t* stg = reinterpret_cast<uint16_t*>(smem + tp.stg_off) + (size_t)grp * kStgBytes;  // 2 buffers
     int stg_step = 0;
     const int bar = 1 + grp;        // named barrier of this warpgroup
-    for (int64_t w = w0 + grp, n = grp; w < w1; w += kExpGroups, n += kExpGroups) {
+    for (int64_t w = w0 + grp, n = grp; w < w1; w += EG, n += EG) {
       const bool seg_last = (w + 1 == w1) || t == T - 1;
-      for (t += kExpGroups; t >= T;) t -= T;
+      for (t += EG; t >= T;) t -= T;
       if (!dead) {
         const bool ok = __all_sync(0xffffffffu, mbar_wait(&full[s], ph, p.timeout_ns));
         if (!ok) {
@@ -506,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&a_full[s]);
-      if ((s += kExpGroups) >= slots) {
+      if ((s += EG) >= slots) {
         s -= slots;
         ph ^= 1u;
       }
@@ -526,7 +534,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       dph_bits ^= 1u << db;
       const uint32_t d_taddr = tmem + (uint32_t)db * tp.d_cols;
       if (!dead) {
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(&d_full[db * kExpGroups + grp], dph, p.timeout_ns));
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(&d_full[db * EG + grp], dph, p.timeout_ns));
         if (!ok) {
           dead = true;
           set_status(p.status, kStatusTimeout);
@@ -631,10 +639,10 @@ int ntok_for(int64_t M) {
   return (int)std::max<int64_t>(16, n);
 }
 
-template <int ES>
+template <int ES, int EG>
 sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtensorMap& map_y, size_t smem,
                        cudaStream_t stream, bool pdl) {
-  auto kern = linear_tc_kernel<ES>;
+  auto kern = linear_tc_kernel<ES, EG>;
   static bool configured[kMaxDevices] = {};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -648,7 +656,7 @@ sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtenso
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)tp.p.G);
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(tc_threads(EG));
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -709,16 +717,29 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   // base alignment + barriers (3 per slot, D handshakes), TMEM address, flags, and (TMA
   // stores of y) the staging tiles, 1024-byte aligned
   tp.y_tma = (h->N % 8 == 0) ? 1 : 0;
-  const size_t ctl_bytes = 8 * (3 * kMaxSlots + kMaxDBufs * (kExpGroups + 1)) + 4 + 4 * kExpGroups + 16;
-  const size_t stg_bytes = tp.y_tma ? (size_t)kExpGroups * 2 * kStgBytes : 0;
-  const size_t tail = 1024 + (ctl_bytes + 1023) / 1024 * 1024 + stg_bytes;
-  // S = slots = A stages in use, an even number: the expander warpgroups take alternate
-  // items, so a slot's previous item belongs to the warpgroup now waiting on it, which
-  // keeps the parity wait on the slot's full barrier exact
-  const int slots = (int)std::min<size_t>(std::min<size_t>(kMaxSlots, (kSmemLimit - tail) / p.slot_bytes),
-                                          (size_t)tp.n_a) &
-                    ~1;
-  if (slots < 2) return SP_ERR_UNSUPPORTED;
+  const size_t ctl_bytes = 8 * (3 * kMaxSlots + kMaxDBufs * (kMaxExpGroups + 1)) + 4 + 4 * kMaxExpGroups + 16;
+  // S = slots = A stages in use, a multiple of the expander warpgroups EG: they take items
+  // round-robin, so a slot's previous item belongs to the warpgroup now waiting on it, which
+  // keeps the parity wait on the slot's full barrier exact.  Three groups where the ring
+  // then holds at least two slots per group (token tiles of up to 64 tokens), else two.
+  int eg = 0, slots = 0;
+  size_t tail = 0;
+  for (const int cand : {kMaxExpGroups, 2}) {
+    if (cand == kMaxExpGroups && tp.ntok > 64) continue;
+    const size_t stg_bytes = tp.y_tma ? (size_t)cand * 2 * kStgBytes : 0;
+    const size_t tl = 1024 + (ctl_bytes + 1023) / 1024 * 1024 + stg_bytes;
+    if (tl >= kSmemLimit) continue;
+    const int sl =
+        (int)std::min<size_t>(std::min<size_t>(kMaxSlots, (kSmemLimit - tl) / p.slot_bytes), (size_t)tp.n_a) /
+        cand * cand;
+    if (sl >= (cand == kMaxExpGroups ? 2 * cand : cand)) {
+      eg = cand;
+      slots = sl;
+      tail = tl;
+      break;
+    }
+  }
+  if (eg == 0) return SP_ERR_UNSUPPORTED;
   p.slots = slots;
   tp.stg_off = (uint32_t)((size_t)slots * p.slot_bytes + (ctl_bytes + 1023) / 1024 * 1024);
   // at least 116 KB so that two CTAs never share an SM (each allocates 512 TMEM columns)
@@ -751,8 +772,12 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   // after an in-place weight update the launch waits for the whole previous grid (no
   // weight copy may start before its writes are visible)
   const bool pdl = !h->weights_written;
-  st = h->esize == 2 ? launch_tc_es<2>(tp, map, map_y, smem, stream, pdl)
-                     : launch_tc_es<1>(tp, map, map_y, smem, stream, pdl);
+  if (eg == kMaxExpGroups)
+    st = h->esize == 2 ? launch_tc_es<2, kMaxExpGroups>(tp, map, map_y, smem, stream, pdl)
+                       : launch_tc_es<1, kMaxExpGroups>(tp, map, map_y, smem, stream, pdl);
+  else
+    st = h->esize == 2 ? launch_tc_es<2, 2>(tp, map, map_y, smem, stream, pdl)
+                       : launch_tc_es<1, 2>(tp, map, map_y, smem, stream, pdl);
   if (st == SP_OK) h->weights_written = 0;
   return st;
 }
