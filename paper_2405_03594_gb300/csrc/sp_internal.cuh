@@ -3,6 +3,8 @@
 // bulk copies, named barriers, global timer).
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -174,6 +176,35 @@ __device__ __forceinline__ void bulk_g2s_hint(void* dst, const void* src, uint32
       "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
 }
+// 1-D bulk copy shared -> global in the issuing thread's bulk async-group.  dst, src and
+// bytes must be multiples of 16.
+__device__ __forceinline__ void bulk_s2g(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(smem_u32(src)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {  // at most N groups still reading shared memory
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy writes of shared memory become visible to the async proxy (TMA, bulk copies)
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// 2-D TMA tile load into shared memory, completing its bytes on `bar`.  The innermost
+// coordinate c0 times the element size must be a multiple of 16 bytes.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+          "r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -255,9 +286,9 @@ __device__ __forceinline__ uint16_t float_to_bf16_bits_rn(float f) {
 sp_status launch_compress(const void* w, const uint8_t* mask, int64_t N, int64_t K, sp_dtype dt, const float* scale,
                           sp_alloc_fn alloc, sp_free_fn free_fn, void* ctx, cudaStream_t stream, sp_matrix** out);
 sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream);
-// allow_cluster: each launch takes the split cluster_cc models fastest for its batch rows:
-// a thread-block cluster over each row block (no workspace needed) or stream-K with
-// split-K partials in the workspace; without it every launch is stream-K.
+// allow_cluster: each launch takes the configuration select_cc picks for its batch rows: a
+// thread-block cluster over each row block (no workspace needed) or stream-K with split-K
+// partials in the workspace; without it every launch is stream-K.
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream, bool allow_cluster = true, uint64_t probe_ns = 0);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
@@ -265,6 +296,7 @@ int cc_kernel_kind(const sp_matrix* h, int64_t M);  // 0 thread-per-row, 1 warp-
 sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
                            cudaStream_t stream);
 size_t workspace_bytes_tc(const sp_matrix* h, int64_t M);
+sp_status tensor_map_encoder(PFN_cuTensorMapEncodeTiled_v12000* out);  // cuTensorMapEncodeTiled, looked up once
 int* device_status_ptr();            // this device's status word (device address)
 uint64_t wait_timeout_ns();          // bounded-wait limit for kernels
 void* dev_alloc(const sp_matrix* h, size_t bytes);

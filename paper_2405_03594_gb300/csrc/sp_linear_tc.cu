@@ -106,16 +106,6 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int c0, int c1, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
-          "r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-}
 // TMA tile store shared -> global (bulk group); rows/columns past the tensor are clipped.
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int c0, int c1) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
@@ -123,17 +113,6 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
                "r"(smem_u32(src)), "r"(c0), "r"(c1)
                : "memory");
 }
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void bulk_wait_read() {  // at most N groups still reading shared memory
-  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// generic-proxy writes of shared memory become visible to the async proxy (TMA)
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row atoms of
 // 1024 bytes stacked along M/N (stride byte offset 1024), atom base 1024-byte aligned.
 __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
@@ -612,26 +591,6 @@ __global__ void __launch_bounds__(tc_threads(EG), 1)
 }
 
 // ------------------------------------------------------------------ host side
-PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
-std::mutex g_encode_mu;
-
-sp_status get_encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
-  std::lock_guard<std::mutex> lk(g_encode_mu);
-  if (!g_encode) {
-    void* fn = nullptr;
-    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
-            cudaSuccess ||
-        q != cudaDriverEntryPointSuccess || !fn) {
-      cudaGetLastError();
-      return SP_ERR_CUDA;
-    }
-    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-  }
-  *out = g_encode;
-  return SP_OK;
-}
-
 int grid_tc(const sp_matrix* h, int64_t W) { return (int)std::min<int64_t>(h->num_sms, W); }
 
 int ntok_for(int64_t M) {
@@ -673,6 +632,26 @@ sp_status launch_tc_es(const TcParams& tp, const CUtensorMap& map, const CUtenso
 
 }  // namespace
 
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::mutex g_encode_mu;
+
+sp_status tensor_map_encoder(PFN_cuTensorMapEncodeTiled_v12000* out) {
+  std::lock_guard<std::mutex> lk(g_encode_mu);
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn) {
+      cudaGetLastError();
+      return SP_ERR_CUDA;
+    }
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  *out = g_encode;
+  return SP_OK;
+}
+
 size_t workspace_bytes_tc(const sp_matrix* h, int64_t M) {
   const int ntok = ntok_for(M);
   const int64_t mt = (M + ntok - 1) / ntok;
@@ -686,7 +665,7 @@ sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   if (!ws || ws_bytes < workspace_bytes_tc(h, M)) return SP_ERR_WORKSPACE;
   if (M > ((int64_t)1 << 31) / kMaxNtok) return SP_ERR_UNSUPPORTED;
   PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-  sp_status st = get_encoder(&encode);
+  sp_status st = tensor_map_encoder(&encode);
   if (st != SP_OK) return st;
   TcParams tp{};
   LinearParams& p = tp.p;
