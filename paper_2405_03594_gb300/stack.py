@@ -110,9 +110,10 @@ class LinearStack:
 
     def launches_per_step(self, M: int, reset: bool = True) -> int:
         """libsp kernels per step: the four sparse linears (as many launches as the library
-        reports for M rows) and four glue kernels per layer, plus the input copy."""
+        reports for M rows) and the glue kernels per layer (four; three at M = 1, where the
+        o linear reads qkv's v block in place), plus the input copy."""
         per_layer = sum(self.mats[n][0].launch_count(M, self.path) for n in SHAPES)
-        return self.layers * (per_layer + 4) + (1 if reset else 0)
+        return self.layers * (per_layer + (3 if M == 1 else 4)) + (1 if reset else 0)
 
     def set_input(self, x: torch.Tensor):
         """Token embeddings [M, 4096] bf16 for the next steps."""
@@ -132,10 +133,14 @@ class LinearStack:
             self.mats["qkv"][l].linear(h, out=qkv, **kw)
             if record is not None:
                 record.append((l, "qkv", h.clone(), qkv.clone()))
-            sp.copy_columns(v, qkv, 2 * D_MODEL, stream=stream)
-            self.mats["o"][l].linear(v, out=o, **kw)
+            # one row of qkv's v block is already a contiguous, 16-byte aligned vector: the o
+            # linear reads it in place; more rows are gathered by one glue launch
+            vin = qkv[:, 2 * D_MODEL:] if M == 1 else v
+            if M != 1:
+                sp.copy_columns(v, qkv, 2 * D_MODEL, stream=stream)
+            self.mats["o"][l].linear(vin, out=o, **kw)
             if record is not None:
-                record.append((l, "o", v.clone(), o.clone()))
+                record.append((l, "o", vin.clone(), o.clone()))
             sp.residual_add(h, o, self.r1[l], stream=stream)
             self.mats["gate_up"][l].linear(h, out=gu, **kw)
             if record is not None:
