@@ -69,6 +69,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_workspace_size.argtypes = [P, I64, ctypes.POINTER(SZ)]
     lib.sp_linear.argtypes = [P, P, I64, P, P, SZ, P]
     lib.sp_linear_ex.argtypes = [P, P, I64, P, P, SZ, ctypes.c_int, P]
+    lib.sp_launch_count.argtypes = [P, I64, ctypes.c_int, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int32)]
     lib.sp_linear_noalloc.argtypes = [P, P, I64, P, P]
     lib.sp_test_expired_wait.argtypes = [P, P, I64, P, P, SZ, ctypes.c_uint32, P]
     lib.sp_masked_update.argtypes = [P, P, ctypes.c_float, P]
@@ -126,9 +127,17 @@ def _check(code: int, where: str):
         raise SpError(code, where)
 
 
-def _stream(stream=None) -> ctypes.c_void_p:
-    s = torch.cuda.current_stream() if stream is None else stream
-    return ctypes.c_void_p(s.cuda_stream)
+# The current stream's raw handle without building a torch.cuda.Stream object per call (a
+# decode step makes ~130 calls; the public route costs a few microseconds of host time each).
+_RAW_STREAM = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
+def _stream(stream=None, device: int | None = None):
+    if stream is not None:
+        return stream.cuda_stream
+    if _RAW_STREAM is not None and device is not None:
+        return _RAW_STREAM(device)
+    return torch.cuda.current_stream().cuda_stream
 
 
 def _ptr(t: torch.Tensor | None) -> ctypes.c_void_p:
@@ -150,6 +159,7 @@ class SparseMatrix:
         self.info = info
         self.n, self.k = int(info.n), int(info.k)
         self.dtype = "int8" if info.dtype == SP_INT8 else "bf16"
+        self.device = int(info.device)
 
     @property
     def handle(self):
@@ -181,8 +191,8 @@ class SparseMatrix:
             out = torch.empty((m, self.n), dtype=torch.bfloat16, device=x.device)
         if workspace is None:
             workspace = workspace_for(self.workspace_size(m), x.device)
-        _check(_lib.sp_linear_ex(self._h, _ptr(x), m, _ptr(out), _ptr(workspace), workspace.numel(), PATHS[path],
-                                 _stream(stream)), "sp_linear")
+        _check(_lib.sp_linear_ex(self._h, x.data_ptr(), m, out.data_ptr(), workspace.data_ptr(), workspace.numel(),
+                                 PATHS[path], _stream(stream, self.device)), "sp_linear")
         return out
 
     def linear_noalloc(self, x: torch.Tensor, out: torch.Tensor, stream=None) -> torch.Tensor:
