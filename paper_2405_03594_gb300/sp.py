@@ -200,7 +200,7 @@ class SparseMatrix:
         callers that cannot allocate device memory; `out` [m, N] bf16 must be given."""
         assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
         assert out.dtype == torch.bfloat16 and out.shape == (x.shape[0], self.n) and out.is_contiguous()
-        _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)), "sp_linear_noalloc")
+        _check(_lib.sp_linear_noalloc(self._h, _ptr(x), x.shape[0], _ptr(out), _stream(stream, self.device)), "sp_linear_noalloc")
         return out
 
     def test_expired_wait(self, x: torch.Tensor, out: torch.Tensor, workspace: torch.Tensor, wait_ms: int,
@@ -229,7 +229,7 @@ class SparseMatrix:
         if workspace is None:
             workspace = workspace_for(self.w8a8_workspace_size(m), qx.device)
         _check(_lib.sp_linear_w8a8(self._h, _ptr(qx), _ptr(sx), m, _ptr(out), _ptr(workspace), workspace.numel(),
-                                   _stream(stream)), "sp_linear_w8a8")
+                                   _stream(stream, self.device)), "sp_linear_w8a8")
         return out
 
     def masked_update(self, grad: torch.Tensor, lr: float, stream=None) -> "SparseMatrix":
@@ -237,7 +237,7 @@ class SparseMatrix:
         the compressed values (Algorithm 1's masked step); grad [N, K] float32 on this
         matrix's device."""
         assert grad.dtype == torch.float32 and grad.shape == (self.n, self.k) and grad.is_contiguous()
-        _check(_lib.sp_masked_update(self._h, _ptr(grad), float(lr), _stream(stream)), "sp_masked_update")
+        _check(_lib.sp_masked_update(self._h, _ptr(grad), float(lr), _stream(stream, self.device)), "sp_masked_update")
         return self
 
     def decompress(self, stream=None) -> torch.Tensor:
@@ -308,21 +308,22 @@ def workspace_for(nbytes: int, device) -> torch.Tensor:
 def copy_columns(out: torch.Tensor, inp: torch.Tensor, col0: int, stream=None) -> torch.Tensor:
     """out[m, :] = inp[m, col0 : col0 + out.shape[1]] (bf16, in a libsp kernel)."""
     M, n = out.shape
-    _check(_lib.sp_copy_columns(_ptr(out), _ptr(inp), M, inp.shape[1], col0, n, _stream(stream)), "sp_copy_columns")
+    _check(_lib.sp_copy_columns(_ptr(out), _ptr(inp), M, inp.shape[1], col0, n, _stream(stream, out.device.index)),
+           "sp_copy_columns")
     return out
 
 
 def residual_add(h: torch.Tensor, a: torch.Tensor, r: torch.Tensor, stream=None) -> torch.Tensor:
     """h = bf16(h + a + r) in place, r broadcast over rows."""
     M, N = h.shape
-    _check(_lib.sp_residual_add(_ptr(h), _ptr(a), _ptr(r), M, N, _stream(stream)), "sp_residual_add")
+    _check(_lib.sp_residual_add(_ptr(h), _ptr(a), _ptr(r), M, N, _stream(stream, h.device.index)), "sp_residual_add")
     return h
 
 
 def mul_halves(out: torch.Tensor, g: torch.Tensor, stream=None) -> torch.Tensor:
     """out = bf16(g[:, :F] * g[:, F:]) with F = out.shape[1]."""
     M, F = out.shape
-    _check(_lib.sp_mul_halves(_ptr(out), _ptr(g), M, F, _stream(stream)), "sp_mul_halves")
+    _check(_lib.sp_mul_halves(_ptr(out), _ptr(g), M, F, _stream(stream, out.device.index)), "sp_mul_halves")
     return out
 
 
@@ -352,7 +353,7 @@ class Chain:
 
     def run(self, stream=None):
         _check(_lib.sp_chain_run(self._ops, self.n_ops, self.m, _ptr(self.workspace), self.workspace.numel(),
-                                 _stream(stream)), "sp_chain_run")
+                                 _stream(stream, self.workspace.device.index)), "sp_chain_run")
 
 
 def check(stream=None):
