@@ -41,6 +41,12 @@ sp_status sp_residual_add(void* h, const void* a, const void* r, int64_t M, int6
  * g[m, F + j]) for j < F; g [M, 2F], out [M, F]; F % 8 == 0. */
 sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* stream);
 
+/* Stack glue, the same product for a gate/up weight whose rows are interleaved (gate_j,
+ * up_j): out[m, j] = bf16(g[m, 2j] * g[m, 2j + 1]) for j < F; g [M, 2F], out [M, F];
+ * F % 8 == 0.  (Library plumbing: the tensor-core path's counterpart of the pair-product
+ * epilogue of sp_linear_epi below.) */
+sp_status sp_mul_pairs(void* out, const void* g, int64_t M, int64_t F, void* stream);
+
 
 /* ---------------------------------------------------------------- chained decode step
  * A chain of sparse linears run by one persistent launch (a decode step through the
@@ -86,6 +92,22 @@ sp_status sp_chain_workspace_size(int64_t m, size_t* bytes);
  * m == 0 or n_ops == 0 returns SP_OK without a launch. */
 sp_status sp_chain_run(const sp_chain_op* ops, int32_t n_ops, int64_t m, void* workspace_dev, size_t workspace_bytes,
                        void* stream);
+
+/* One sparse linear (Sec. 2.4.2) with the stack's glue folded into its output: y =
+ * epilogue(x . (W o Mask)^T) with the epilogues of sp_chain_epilogue -- SP_EPI_STORE as
+ * sp_linear; SP_EPI_RESIDUAL y[m, n] = bf16((y[m, n] + bf16(acc)) + r[n]) in place;
+ * SP_EPI_PAIR_PRODUCT y[m, j] = bf16(bf16(acc_2j) * bf16(acc_2j+1)), y [m, N/2] (N even).
+ * The epilogue's results equal those of sp_linear followed by sp_residual_add or
+ * sp_mul_pairs (bitwise, for the same kernel and batch).  x [m, K] and y are bf16,
+ * contiguous and 16-byte aligned; r is bf16 [N] for SP_EPI_RESIDUAL, else NULL; the
+ * workspace is as for sp_linear (sp_workspace_size bytes, zero-filled once, calls that
+ * share it ordered on one stream).  Runs on the CUDA-core kernels: where the automatic path
+ * takes the tensor-core kernel for m rows the call returns SP_ERR_UNSUPPORTED without a
+ * launch, and the caller uses sp_linear and the glue call instead.  Other errors as
+ * sp_linear, and SP_ERR_INVALID_ARG for an unknown epilogue, a missing r or an odd N with
+ * the pair product. */
+sp_status sp_linear_epi(const sp_matrix* h, const void* x, int64_t m, void* y, int32_t epilogue, const void* r,
+                        void* workspace_dev, size_t workspace_bytes, void* stream);
 
 #ifdef __cplusplus
 }

@@ -5,6 +5,7 @@
 #include <algorithm>
 #include <mutex>
 
+#include "../../include/sp_stack.h"
 #include "sp_internal.cuh"
 
 namespace sp {
@@ -134,6 +135,33 @@ sp_status sp_linear_ex(const sp_matrix* h, const void* x_dev, int64_t m, void* y
                             workspace_bytes, (cudaStream_t)stream);
   return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
                           workspace_bytes, (cudaStream_t)stream);
+}
+
+sp_status sp_linear_epi(const sp_matrix* h, const void* x_dev, int64_t m, void* y_dev, int32_t epilogue,
+                        const void* r_dev, void* workspace_dev, size_t workspace_bytes, void* stream) {
+  if (!live(h)) return SP_ERR_BAD_HANDLE;
+  if (m < 0) return SP_ERR_INVALID_ARG;
+  if (epilogue != SP_EPI_STORE && epilogue != SP_EPI_RESIDUAL && epilogue != SP_EPI_PAIR_PRODUCT)
+    return SP_ERR_INVALID_ARG;
+  if (epilogue == SP_EPI_RESIDUAL && !r_dev) return SP_ERR_INVALID_ARG;
+  if (epilogue == SP_EPI_PAIR_PRODUCT && h->N % 2 != 0) return SP_ERR_INVALID_ARG;
+  if (m == 0) return SP_OK;
+  if (!x_dev || !y_dev) return SP_ERR_INVALID_ARG;
+  if (!aligned16(x_dev) || !aligned16(y_dev) || (workspace_dev && !aligned16(workspace_dev)) ||
+      (r_dev && (reinterpret_cast<uintptr_t>(r_dev) & 1u)))
+    return SP_ERR_ALIGNMENT;
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return SP_ERR_CUDA;
+  }
+  if (dev != h->device) return SP_ERR_INVALID_ARG;
+  if (!workspace_dev || workspace_bytes < std::max(workspace_bytes_cc(h, m), workspace_bytes_tc(h, m)))
+    return SP_ERR_WORKSPACE;
+  if (uses_tensor_cores(h, m, SP_PATH_AUTO)) return SP_ERR_UNSUPPORTED;
+  return launch_linear_cc(h, static_cast<const uint16_t*>(x_dev), m, static_cast<uint16_t*>(y_dev), workspace_dev,
+                          workspace_bytes, (cudaStream_t)stream, true, 0, epilogue,
+                          static_cast<const uint16_t*>(r_dev));
 }
 
 sp_status sp_launch_count(const sp_matrix* h, int64_t m, sp_path path, int64_t* launches, int32_t* kernel) {

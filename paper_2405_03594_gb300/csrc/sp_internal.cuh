@@ -80,6 +80,8 @@ struct LinearParams {
   uint32_t comb_off;    // warp-per-chunk kernel: shared-memory offset of the warps' partials
   uint64_t probe_ns;    // 0, except in the failure-path test: consumer warp 0 of CTA 0 first
                         // waits this long on a barrier that nothing completes
+  int32_t epi;          // CUDA-core kernels: the output epilogue (sp_chain_epilogue; 0 = store)
+  const uint16_t* r;    // SP_EPI_RESIDUAL: bf16 [N] residual vector
 };
 
 // Workspace layout, fixed per device so that calls with different grids can share it:
@@ -290,7 +292,8 @@ sp_status launch_decompress(const sp_matrix* h, void* w_out, cudaStream_t stream
 // thread-block cluster over each row block (no workspace needed) or stream-K with split-K
 // partials in the workspace; without it every launch is stream-K.
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream, bool allow_cluster = true, uint64_t probe_ns = 0);
+                           cudaStream_t stream, bool allow_cluster = true, uint64_t probe_ns = 0, int32_t epi = 0,
+                           const uint16_t* r = nullptr);
 size_t workspace_bytes_cc(const sp_matrix* h, int64_t M);
 int cc_kernel_kind(const sp_matrix* h, int64_t M);  // 0 thread-per-row, 1 warp-per-chunk, -1 none fits
 sp_status launch_linear_tc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,

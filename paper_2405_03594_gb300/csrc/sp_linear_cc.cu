@@ -23,6 +23,7 @@
 //                    (deterministic split-K).
 #include <algorithm>
 
+#include "../../include/sp_stack.h"
 #include "sp_cc_common.cuh"
 
 namespace sp {
@@ -146,6 +147,39 @@ __device__ __forceinline__ void produce(const LinearParams& p, uint8_t* smem, ui
 //    last), and the last of the row block's CTAs to arrive sums the partials in CTA
 //    order (deterministic) and writes y.
 // All consumer threads (kConsumerWarps warps) call this together.
+// Output of row n for the batch rows from its FP32 sums v (INT8: times the row's scale sc)
+// through the launch's epilogue (the definitions of sp_chain_epilogue): store; residual,
+// y = bf16((y + bf16(v sc)) + r[n]) in place; pair product of rows 2j and 2j+1 into y [m, N/2].
+// All 32 lanes of a warp call it together with consecutive rows (the pair product takes the
+// odd row's value from the neighbouring lane); rows past N write nothing.
+template <int M>
+__device__ __forceinline__ void write_row(const LinearParams& p, int64_t n, const float (&v)[M], float sc) {
+  const bool in = n < p.N;
+  if (p.epi == SP_EPI_PAIR_PRODUCT) {
+    const int64_t ldy = p.N >> 1;
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      const uint32_t g = in ? float_to_bf16_bits_rn(v[m] * sc) : 0u;
+      const uint32_t u = __shfl_xor_sync(0xffffffffu, g, 1);
+      if (in && (n & 1) == 0)
+        p.y[(int64_t)m * ldy + (n >> 1)] = float_to_bf16_bits_rn(bf16_bits_to_float(g) * bf16_bits_to_float(u));
+    }
+  } else if (in) {
+    if (p.epi == SP_EPI_RESIDUAL) {
+      const float rv = bf16_bits_to_float(p.r[n]);
+#pragma unroll
+      for (int m = 0; m < M; ++m) {
+        uint16_t* yp = p.y + (int64_t)m * p.N + n;
+        const float a = bf16_bits_to_float(float_to_bf16_bits_rn(v[m] * sc));
+        *yp = float_to_bf16_bits_rn((bf16_bits_to_float(__ldcg(reinterpret_cast<const unsigned short*>(yp))) + a) + rv);
+      }
+    } else {
+#pragma unroll
+      for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(v[m] * sc);
+    }
+  }
+}
+
 template <int M, int ES, bool CL>
 __device__ __forceinline__ void row_block_end(const LinearParams& p, uint8_t* smem, volatile int* s_flag,
                                               const float (&acc)[M], int64_t rb, bool complete, int my_slot,
@@ -183,17 +217,11 @@ __device__ __forceinline__ void row_block_end(const LinearParams& p, uint8_t* sm
             for (int m = 0; m < M; ++m) sum[m] += v[u][m];
           }
       }
-      if (n < p.N) {
-#pragma unroll
-        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
-      }
+      write_row<M>(p, n, sum, sc);
     }
     cluster_sync_all();
   } else if (complete) {
-    if (n < p.N) {
-#pragma unroll
-      for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(acc[m] * sc);
-    }
+    write_row<M>(p, n, acc, sc);
   } else {
     float* wsp = p.ws + ((int64_t)blockIdx.x * 2 + my_slot) * (kRows * kMaxTokens);
 #pragma unroll
@@ -236,10 +264,7 @@ __device__ __forceinline__ void row_block_end(const LinearParams& p, uint8_t* sm
             for (int m = 0; m < M; ++m) sum[m] += part[u][m];
           }
       }
-      if (n < p.N) {
-#pragma unroll
-        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(sum[m] * sc);
-      }
+      write_row<M>(p, n, sum, sc);
       if (tid == 0) atomicExch(ctr, 0);
     }
     named_bar_sync(1, kConsumerWarps * 32);
@@ -350,14 +375,44 @@ struct FlushCtl {
 // Rows 4*lane + i of row block rb: y = bf16(s * scale)
 template <int M, int ES>
 __device__ __forceinline__ void store_rows(const LinearParams& p, const float (&s)[4][M], int64_t rb, int lane) {
+  // rows 4l .. 4l+3 of this lane: the pairs (4l, 4l+1) and (4l+2, 4l+3) of the pair product
+  // are both in the lane
   const int64_t n0 = rb * kRows + 4 * lane;
+  float sc[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) sc[i] = (ES == 1 && n0 + i < p.N) ? p.scale[n0 + i] : 1.f;
+  if (p.epi == SP_EPI_PAIR_PRODUCT) {
+    const int64_t ldy = p.N >> 1;
+#pragma unroll
+    for (int i = 0; i < 4; i += 2) {
+      const int64_t n = n0 + i;
+      if (n < p.N) {
+#pragma unroll
+        for (int m = 0; m < M; ++m) {
+          const float g = bf16_bits_to_float(float_to_bf16_bits_rn(s[i][m] * sc[i]));
+          const float u = bf16_bits_to_float(float_to_bf16_bits_rn(s[i + 1][m] * sc[i + 1]));
+          p.y[(int64_t)m * ldy + (n >> 1)] = float_to_bf16_bits_rn(g * u);
+        }
+      }
+    }
+    return;
+  }
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int64_t n = n0 + i;
     if (n < p.N) {
-      const float sc = ES == 1 ? p.scale[n] : 1.f;
+      if (p.epi == SP_EPI_RESIDUAL) {
+        const float rv = bf16_bits_to_float(p.r[n]);
 #pragma unroll
-      for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(s[i][m] * sc);
+        for (int m = 0; m < M; ++m) {
+          uint16_t* yp = p.y + (int64_t)m * p.N + n;
+          const float a = bf16_bits_to_float(float_to_bf16_bits_rn(s[i][m] * sc[i]));
+          *yp = float_to_bf16_bits_rn((bf16_bits_to_float(__ldcg(reinterpret_cast<const unsigned short*>(yp))) + a) + rv);
+        }
+      } else {
+#pragma unroll
+        for (int m = 0; m < M; ++m) p.y[(int64_t)m * p.N + n] = float_to_bf16_bits_rn(s[i][m] * sc[i]);
+      }
     }
   }
 }
@@ -822,7 +877,8 @@ size_t workspace_bytes_cc(const sp_matrix* h, int64_t /*M*/) {
 }
 
 sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uint16_t* y, void* ws, size_t ws_bytes,
-                           cudaStream_t stream, bool allow_cluster, uint64_t probe_ns) {
+                           cudaStream_t stream, bool allow_cluster, uint64_t probe_ns, int32_t epi,
+                           const uint16_t* r) {
   // the configuration depends on the batch rows of a launch: full launches of kMaxTokens
   // rows and one ragged tail; the workspace is checked before the first launch
   const bool probe = probe_ns != 0;
@@ -849,6 +905,9 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
   p.ws = ws ? reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ws) + ws_counter_bytes(h->num_sms)) : nullptr;
   p.timeout_ns = wait_timeout_ns();
   p.probe_ns = probe_ns;
+  p.epi = epi;
+  p.r = r;
+  const int64_t ldy = epi == SP_EPI_PAIR_PRODUCT ? h->N / 2 : h->N;
   p.chunk_region = (uint32_t)((h->max_chunk + 127) / 128 * 128);
   for (int64_t m0 = 0; m0 < M; m0 += kMaxTokens) {
     const int Mt = (int)std::min<int64_t>(kMaxTokens, M - m0);
@@ -859,7 +918,7 @@ sp_status launch_linear_cc(const sp_matrix* h, const uint16_t* x, int64_t M, uin
     p.cluster = S;
     p.G = S > 1 ? h->RB * S : grid_cc(h);
     p.x = x + m0 * h->K;
-    p.y = y + m0 * h->N;
+    p.y = y + m0 * ldy;
     p.slot_bytes = pl.slot_bytes;
     p.slots = pl.slots;
     p.comb_off = pl.comb_off;

@@ -70,6 +70,24 @@ __global__ void mul_halves_kernel(uint4* __restrict__ out, const uint4* __restri
   }
 }
 
+// out[m, j] = bf16(g[m, 2j] * g[m, 2j + 1]): eight outputs per thread from two 16-byte
+// loads of g (interleaved gate/up rows' outputs).
+__global__ void mul_pairs_kernel(uint4* __restrict__ out, const uint4* __restrict__ g, int64_t M, int64_t f8,
+                                 bool early_release) {
+  glue_begin(early_release);
+  const int64_t total = M * f8;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t m = i / f8, j = i % f8;
+    const uint4 a = g[m * 2 * f8 + 2 * j], b = g[m * 2 * f8 + 2 * j + 1];
+    uint4 o;
+    o.x = pack2(lo_f(a.x) * hi_f(a.x), lo_f(a.y) * hi_f(a.y));
+    o.y = pack2(lo_f(a.z) * hi_f(a.z), lo_f(a.w) * hi_f(a.w));
+    o.z = pack2(lo_f(b.x) * hi_f(b.x), lo_f(b.y) * hi_f(b.y));
+    o.w = pack2(lo_f(b.z) * hi_f(b.z), lo_f(b.w) * hi_f(b.w));
+    out[i] = o;
+  }
+}
+
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 template <typename... Params, typename... Args>
@@ -123,6 +141,15 @@ sp_status sp_mul_halves(void* out, const void* g, int64_t M, int64_t F, void* st
   if (!al16(out) || !al16(g)) return SP_ERR_ALIGNMENT;
   if (M == 0 || F == 0) return SP_OK;
   return launch_glue(mul_halves_kernel, M * F / 8, (cudaStream_t)stream, (uint4*)out, (const uint4*)g, M, F / 8,
+                     M == 1);
+}
+
+sp_status sp_mul_pairs(void* out, const void* g, int64_t M, int64_t F, void* stream) {
+  if (!out || !g || M < 0 || F < 0) return SP_ERR_INVALID_ARG;
+  if (F % 8) return SP_ERR_UNSUPPORTED;
+  if (!al16(out) || !al16(g)) return SP_ERR_ALIGNMENT;
+  if (M == 0 || F == 0) return SP_OK;
+  return launch_glue(mul_pairs_kernel, M * F / 8, (cudaStream_t)stream, (uint4*)out, (const uint4*)g, M, F / 8,
                      M == 1);
 }
 

@@ -23,11 +23,13 @@ STATUS = {
     0: "SP_OK", 1: "SP_ERR_INVALID_ARG", 2: "SP_ERR_UNSUPPORTED", 3: "SP_ERR_ALIGNMENT", 4: "SP_ERR_CUDA",
     5: "SP_ERR_OUT_OF_MEMORY", 6: "SP_ERR_TIMEOUT", 7: "SP_ERR_BAD_HANDLE", 8: "SP_ERR_WORKSPACE",
 }
+SP_ERR_UNSUPPORTED = 2
 # every function declared in include/sp.h and include/sp_stack.h
 EXPORTS = ["sp_compress", "sp_decompress", "sp_workspace_size", "sp_linear", "sp_linear_ex", "sp_launch_count",
            "sp_linear_noalloc", "sp_test_expired_wait", "sp_masked_update", "sp_linear_w8a8", "sp_w8a8_workspace_size",
            "sp_clone", "sp_free", "sp_info", "sp_copy_out", "sp_check", "sp_status_string",
-           "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_chain_workspace_size", "sp_chain_run"]
+           "sp_copy_columns", "sp_residual_add", "sp_mul_halves", "sp_mul_pairs", "sp_chain_workspace_size",
+           "sp_chain_run", "sp_linear_epi"]
 
 
 KERNELS = {0: "", 1: "linear_cc_kernel", 2: "linear_ccw_kernel", 3: "linear_tc_kernel"}  # SP_KERNEL_*
@@ -83,6 +85,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.sp_copy_columns.argtypes = [P, P, I64, I64, I64, I64, P]
     lib.sp_residual_add.argtypes = [P, P, P, I64, I64, P]
     lib.sp_mul_halves.argtypes = [P, P, I64, I64, P]
+    lib.sp_mul_pairs.argtypes = [P, P, I64, I64, P]
+    lib.sp_linear_epi.argtypes = [P, P, I64, P, ctypes.c_int32, P, P, SZ, P]
     lib.sp_chain_workspace_size.argtypes = [I64, ctypes.POINTER(SZ)]
     lib.sp_chain_run.argtypes = [ctypes.POINTER(SpChainOp), ctypes.c_int32, I64, P, SZ, P]
     lib.sp_status_string.argtypes = [ctypes.c_int]
@@ -194,6 +198,26 @@ class SparseMatrix:
         _check(_lib.sp_linear_ex(self._h, x.data_ptr(), m, out.data_ptr(), workspace.data_ptr(), workspace.numel(),
                                  PATHS[path], _stream(stream, self.device)), "sp_linear")
         return out
+
+    def linear_epi(self, x: torch.Tensor, out: torch.Tensor, epilogue: str, r: torch.Tensor | None = None,
+                   workspace: torch.Tensor | None = None, stream=None) -> bool:
+        """sp_linear_epi: out = epilogue(x . (W o Mask)^T) with "store", "residual" (out updated
+        in place with the bf16 vector r [N]) or "pair_product" (out [m, N/2]).  Returns False,
+        launching nothing, where the batch would run on the tensor-core kernel (the caller
+        then uses linear() and the glue call)."""
+        assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == self.k and x.is_contiguous()
+        m = x.shape[0]
+        ny = self.n // 2 if epilogue == "pair_product" else self.n
+        assert out.dtype == torch.bfloat16 and out.shape == (m, ny) and out.is_contiguous()
+        if workspace is None:
+            workspace = workspace_for(self.workspace_size(m), x.device)
+        code = _lib.sp_linear_epi(self._h, x.data_ptr(), m, out.data_ptr(), EPILOGUES[epilogue],
+                                  0 if r is None else r.data_ptr(), workspace.data_ptr(), workspace.numel(),
+                                  _stream(stream, self.device))
+        if code == SP_ERR_UNSUPPORTED:  # a tensor-core batch
+            return False
+        _check(code, "sp_linear_epi")
+        return True
 
     def linear_noalloc(self, x: torch.Tensor, out: torch.Tensor, stream=None) -> torch.Tensor:
         """sp_linear_noalloc: the decode kernel with the library's own static scratch, for
@@ -318,6 +342,13 @@ def residual_add(h: torch.Tensor, a: torch.Tensor, r: torch.Tensor, stream=None)
     M, N = h.shape
     _check(_lib.sp_residual_add(_ptr(h), _ptr(a), _ptr(r), M, N, _stream(stream, h.device.index)), "sp_residual_add")
     return h
+
+
+def mul_pairs(out: torch.Tensor, g: torch.Tensor, stream=None) -> torch.Tensor:
+    """out = bf16(g[:, 0::2] * g[:, 1::2]) with F = out.shape[1] (interleaved gate/up rows)."""
+    M, F = out.shape
+    _check(_lib.sp_mul_pairs(_ptr(out), _ptr(g), M, F, _stream(stream, out.device.index)), "sp_mul_pairs")
+    return out
 
 
 def mul_halves(out: torch.Tensor, g: torch.Tensor, stream=None) -> torch.Tensor:

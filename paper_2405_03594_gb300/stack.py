@@ -70,19 +70,28 @@ def _layer_mats(layers: int, host, host_layers, dev, interleave_gate_up: bool) -
     return {name: [one[name]] + [one[name].clone() for _ in range(layers - 1)] for name in SHAPES}
 
 
+def _must(ran: bool):
+    if not ran:  # fuses() chose the epilogue path for a batch that the library runs on tensor cores
+        raise RuntimeError("sp_linear_epi declined a batch the stack expected to fuse")
+
+
 class LinearStack:
     """host: one layer's inputs, copied to every layer; host_layers: each layer's own inputs
-    (then `layers` is their count)."""
+    (then `layers` is their count).  fused (automatic path only): the gate/up weight holds
+    interleaved rows and, for batches that run on the CUDA-core kernels, the residual adds and
+    the gate * up product are the linears' epilogues (sp_linear_epi); tensor-core batches keep
+    the separate glue launches (sp_residual_add, sp_mul_pairs)."""
 
     def __init__(self, layers: int = 32, pct: int = 70, int8: bool = True, max_m: int = 64, seed: int = 0,
-                 device=None, host=None, path: str = "auto", host_layers=None):
+                 device=None, host=None, path: str = "auto", host_layers=None, fused: bool = True):
         self.dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
         if host_layers is not None:
             layers = len(host_layers)
         self.layers, self.max_m, self.path = layers, max_m, path
+        self.fused = fused and path == "auto"
         self.host = None if host_layers is not None else (host_layer(pct, int8, seed) if host is None else host)
         self.host_layers = host_layers
-        self.mats = _layer_mats(layers, self.host, host_layers, self.dev, False)
+        self.mats = _layer_mats(layers, self.host, host_layers, self.dev, self.fused)
         g = synth.rng(seed, 0, 9, synth.STREAM_RESID)
         r = synth.activations(2 * layers, D_MODEL, g)
         rt = torch.from_numpy(r.view(np.int16)).to(self.dev).view(torch.bfloat16)
@@ -105,15 +114,26 @@ class LinearStack:
         return sum(int(m.info.bytes) + int(m.info.scale_bytes) for n in SHAPES for m in self.mats[n])
 
     def host_of(self, layer: int, name: str):
-        """Host (values, mask, scale) of `name` in `layer`."""
-        return (self.host_layers[layer] if self.host_layers is not None else self.host)[name]
+        """Host (values, mask, scale) of `name` in `layer` (gate/up with interleaved rows when
+        fused)."""
+        vals, mask, s = (self.host_layers[layer] if self.host_layers is not None else self.host)[name]
+        if self.fused and name == "gate_up":
+            vals, mask = interleave_rows(vals, D_FF), interleave_rows(mask, D_FF)
+            s = None if s is None else interleave_rows(s, D_FF)
+        return vals, mask, s
+
+    def fuses(self, M: int) -> bool:
+        """Whether a step of M rows folds the residual adds and gate * up into the linears."""
+        return self.fused and all(self.mats[n][0].kernel_name(M) != "linear_tc_kernel" for n in SHAPES)
 
     def launches_per_step(self, M: int, reset: bool = True) -> int:
         """libsp kernels per step: the four sparse linears (as many launches as the library
-        reports for M rows) and the glue kernels per layer (four; three at M = 1, where the
-        o linear reads qkv's v block in place), plus the input copy."""
+        reports for M rows) and the glue kernels per layer: the v-block copy (none at M = 1,
+        where the o linear reads it in place), and the two residual adds and gate * up unless
+        they are the linears' epilogues; plus the input copy."""
         per_layer = sum(self.mats[n][0].launch_count(M, self.path) for n in SHAPES)
-        return self.layers * (per_layer + (3 if M == 1 else 4)) + (1 if reset else 0)
+        glue = (0 if M == 1 else 1) + (0 if self.fuses(M) else 3)
+        return self.layers * (per_layer + glue) + (1 if reset else 0)
 
     def set_input(self, x: torch.Tensor):
         """Token embeddings [M, 4096] bf16 for the next steps."""
@@ -123,33 +143,50 @@ class LinearStack:
 
     def step(self, M: int, record=None, stream=None, reset: bool = False):
         """One decode step for the first M rows of self.h (in place); with reset=True it
-        starts from the saved input (set_input).  If `record` is a list, each linear's
-        (layer, shape, input, output) copies are appended to it."""
+        starts from the saved input (set_input).  If `record` is a list, each linear appends
+        (layer, shape, input, output, epilogue, h before the linear) copies: epilogue "store"
+        (output = the linear's result), "residual" (output = h after it, in place) or
+        "pair_product" (output = gate * up)."""
         kw = dict(workspace=self.ws, path=self.path, stream=stream)
         h, qkv, v, o, gu, a, d = (t[:M] for t in (self.h, self.qkv, self.v, self.o, self.gu, self.a, self.d))
+        fuse = self.fuses(M)
         if reset:
             sp.copy_columns(h, self.x0[:M], 0, stream=stream)
         for l in range(self.layers):
             self.mats["qkv"][l].linear(h, out=qkv, **kw)
             if record is not None:
-                record.append((l, "qkv", h.clone(), qkv.clone()))
+                record.append((l, "qkv", h.clone(), qkv.clone(), "store", None))
             # one row of qkv's v block is already a contiguous, 16-byte aligned vector: the o
             # linear reads it in place; more rows are gathered by one glue launch
             vin = qkv[:, 2 * D_MODEL:] if M == 1 else v
             if M != 1:
                 sp.copy_columns(v, qkv, 2 * D_MODEL, stream=stream)
-            self.mats["o"][l].linear(vin, out=o, **kw)
+            self._residual("o", l, vin, o, h, self.r1[l], fuse, record, stream)
+            if fuse:
+                hb = h.clone() if record is not None else None
+                _must(self.mats["gate_up"][l].linear_epi(h, a, "pair_product", workspace=self.ws, stream=stream))
+                if record is not None:
+                    record.append((l, "gate_up", hb, a.clone(), "pair_product", None))
+            else:
+                self.mats["gate_up"][l].linear(h, out=gu, **kw)
+                if record is not None:
+                    record.append((l, "gate_up", h.clone(), gu.clone(), "store", None))
+                (sp.mul_pairs if self.fused else sp.mul_halves)(a, gu, stream=stream)
+            self._residual("down", l, a, d, h, self.r2[l], fuse, record, stream)
+
+    def _residual(self, name, l, x, tmp, h, r, fuse, record, stream):
+        """h <- bf16((h + bf16(linear(x))) + r): the linear's epilogue, or a linear into tmp
+        and the glue add."""
+        hb = h.clone() if record is not None else None
+        if fuse:
+            _must(self.mats[name][l].linear_epi(x, h, "residual", r, workspace=self.ws, stream=stream))
             if record is not None:
-                record.append((l, "o", vin.clone(), o.clone()))
-            sp.residual_add(h, o, self.r1[l], stream=stream)
-            self.mats["gate_up"][l].linear(h, out=gu, **kw)
-            if record is not None:
-                record.append((l, "gate_up", h.clone(), gu.clone()))
-            sp.mul_halves(a, gu, stream=stream)
-            self.mats["down"][l].linear(a, out=d, **kw)
-            if record is not None:
-                record.append((l, "down", a.clone(), d.clone()))
-            sp.residual_add(h, d, self.r2[l], stream=stream)
+                record.append((l, name, x.clone(), h.clone(), "residual", hb))
+            return
+        self.mats[name][l].linear(x, out=tmp, workspace=self.ws, path=self.path, stream=stream)
+        if record is not None:
+            record.append((l, name, x.clone(), tmp.clone(), "store", hb))
+        sp.residual_add(h, tmp, r, stream=stream)
 
     def capture(self, M: int) -> torch.cuda.CUDAGraph:
         """One decode step from the saved input, recorded as a single CUDA graph."""

@@ -104,6 +104,9 @@ def test_handle_checks(lib):
     assert lib.sp_masked_update(None, P(1 << 20), ctypes.c_float(0.1), None) == 7
     assert lib.sp_linear_w8a8(None, P(1 << 20), P(1 << 20), 1, P(1 << 20), None, 0, None) == 7
     assert lib.sp_w8a8_workspace_size(None, 4, ctypes.byref(sz)) == 7
+    assert lib.sp_linear_epi(None, P(1 << 20), 1, P(1 << 20), 0, None, None, 0, None) == 7
+    assert lib.sp_mul_pairs(None, P(1 << 20), 1, 8, None) == 1  # no output
+    assert lib.sp_mul_pairs(P(1 << 20), P(1 << 20), 1, 12, None) == 2  # F % 8 != 0
     # a pointer that is not a handle is rejected by its magic word
     junk = (ctypes.c_uint32 * 64)()
     assert lib.sp_info(ctypes.cast(junk, P), None) == 7

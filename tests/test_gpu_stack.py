@@ -1,6 +1,7 @@
-"""The linear-stack decode step (INT8 weights, 70%): every sparse linear is checked
-against the float64 oracle on the GPU's own inputs, the glue against the oracle's glue,
-and a CUDA-graph replay against the eager step."""
+"""The linear-stack decode step (INT8 weights, 70%): every sparse linear (with its fused
+residual or gate * up epilogue where the batch runs on the CUDA cores) is checked against the
+float64 oracle on the GPU's own inputs, the glue against the oracle's glue, and a CUDA-graph
+replay against the eager step."""
 import numpy as np
 import pytest
 
@@ -35,15 +36,14 @@ def test_each_linear_matches_oracle_on_gpu_inputs(stack, oracle, M):
     sp.check()
     assert len(rec) == 4 * stack.layers
     rows_rng = np.random.default_rng(M)
-    for layer, name, inp, out in rec:
-        q, mask, s = stack.host[name]
-        xin = _bits(inp)
-        y = gu.bf16_from_dev(out)
-        assert np.isfinite(y).all()
-        N = q.shape[0]
-        rows = np.arange(N) if M <= 4 else np.sort(rows_rng.choice(N, 256, replace=False))
-        ref = oracle.linear_int8(xin, q[rows], mask[rows], s[rows])
-        gu.assert_close(y[:, rows], ref, f"layer {layer} {name} M={M}")
+    for item in rec:
+        layer, name = item[0], item[1]
+        N = stack.host_of(layer, name)[0].shape[0]
+        rows = None if M <= 4 else np.sort(rows_rng.choice(N, 256, replace=False))
+        pairs = None if M <= 4 else np.sort(rows_rng.choice(N // 2, 128, replace=False))
+        gu.check_stack_record(oracle, stack, item, rows=rows, sample_pairs=pairs, what=f"layer {layer} {name} M={M}")
+    # batches on the CUDA-core kernels fold the glue into the linears' epilogues
+    assert {e[4] for e in rec} == ({"store", "residual", "pair_product"} if stack.fuses(M) else {"store"})
 
 
 def test_glue_matches_oracle(stack, oracle):
