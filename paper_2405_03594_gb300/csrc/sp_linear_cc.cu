@@ -5,8 +5,11 @@
 // memory onto the chip and are expanded there by their bitmask; decode is bound
 // by those bytes, Sec. 2.4, 3.4).
 //
-// Launch: G persistent CTAs (4 per SM), each owning a contiguous run of chunks in
-// storage order (stream-K), so every CTA streams one linear byte range.
+// Launch: each row block split over the S CTAs of a thread-block cluster (partials summed
+// over distributed shared memory), or -- when not even two CTAs per row block fit -- G
+// CTAs each owning a contiguous run of chunks in storage order (stream-K), so every CTA
+// streams one linear byte range.  Four CTAs per SM, six for one-row warp-per-chunk
+// cluster launches (cluster_cc and select_cc below).
 //   warp 4, lane 0   producer: one cp.async.bulk per chunk (+ one copy of
 //                    x[m, 64t : 64t+64) per batch row) into a ring of `slots`
 //                    shared-memory slots, each guarded by a full/empty mbarrier
@@ -17,10 +20,12 @@
 //                    independent chains: columns 0-31 and 32-63), gathers
 //                    x[m, 64t+j] from lane j%32 by shuffle (two batch rows per
 //                    register), and accumulates with the FP32-accumulating bf16 FMA.
-//                    At a row-block end the 128 rows are written (bf16, RNE), or --
-//                    when the row block is shared with other CTAs -- stored as an FP32
-//                    partial and summed in CTA order by the last CTA to arrive
-//                    (deterministic split-K).
+//                    At a row-block end the 128 rows are written (bf16, RNE, through
+//                    the launch's output epilogue), or -- when the row block is shared
+//                    with other CTAs outside a cluster -- stored as an FP32 partial and
+//                    summed in CTA order by the last CTA to arrive (deterministic
+//                    split-K).  The warp-per-chunk kernel (M <= 4) is described at its
+//                    definition below.
 #include <algorithm>
 
 #include "../../include/sp_stack.h"
