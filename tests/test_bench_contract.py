@@ -264,3 +264,22 @@ def test_profile_and_square_sections_report_failures_instead_of_raising():
     assert "error" in pr and sum(pr["profile"]) == 70 * b.LAYERS
     sq = b.square_section(args)
     assert "error" in sq and sq["points"] == {}
+
+
+def test_kernel_source_hash_ignores_comments_but_not_code(tmp_path, monkeypatch):
+    """The traffic record stays valid across comment edits of a kernel's sources and is
+    discarded by any code edit."""
+    import shutil
+
+    b = _bench_module()
+    root = tmp_path / "repo"
+    shutil.copytree(os.path.join(b.ROOT, "paper_2405_03594_gb300", "csrc"), root / "paper_2405_03594_gb300" / "csrc")
+    shutil.copytree(os.path.join(b.ROOT, "include"), root / "include")
+    monkeypatch.setattr(b, "ROOT", str(root))
+    base = b.kernel_source_hash("linear_ccw_kernel")
+    src = root / "paper_2405_03594_gb300" / "csrc" / "sp_linear_cc.cu"
+    text = src.read_text()
+    src.write_text("// a new comment line\n" + text.replace("// Launch:", "/* block comment */ // Launch:", 1))
+    assert b.kernel_source_hash("linear_ccw_kernel") == base
+    src.write_text(text.replace("constexpr int kCtasPerSm = 4;", "constexpr int kCtasPerSm = 5;", 1))
+    assert b.kernel_source_hash("linear_ccw_kernel") != base
