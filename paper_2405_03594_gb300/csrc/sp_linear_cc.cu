@@ -48,6 +48,10 @@ constexpr size_t kSmemOptIn = 54 * 1024;
 // registers and keep four.
 constexpr int kCtasPerSmM1 = 6;
 constexpr size_t kSmemBudgetM1 = 37 * 1024;
+// Where four slots of the largest chunk do not fit that budget (50 % sparsity: ~9.2 KB
+// chunks), one-row cluster launches run five CTAs per SM (72 registers, no spills; 44 KB).
+constexpr int kCtasPerSmM1b = 5;
+constexpr size_t kSmemBudgetM1b = 44 * 1024;
 
 // CTA's work items [w0, w1): a contiguous run of chunks (stream-K), or -- in cluster
 // mode -- K-tiles [r*T/S, (r+1)*T/S) of the row block of its cluster (r = its rank).
@@ -564,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, OCC) linear_ccw_kernel(const LinearP
   volatile int* s_flag = reinterpret_cast<volatile int*>(empty + p.slots);
   volatile int* tag = s_flag + 4;
   float* comb = reinterpret_cast<float*>(smem + p.comb_off);  // [2][kConsumerWarps][M][kRows]
-  FlushCtl* fctl = reinterpret_cast<FlushCtl*>(comb + 2 * kConsumerWarps * M * kRows);
+  FlushCtl* fctl = reinterpret_cast<FlushCtl*>(comb + (CL ? 1 : 2) * kConsumerWarps * M * kRows);
   // PROBE (the failure-path test only): a barrier that nothing completes, in the unused upper
   // half of the 16-byte flag area (8-byte aligned: it follows the mbarrier arrays)
   uint64_t* probe = reinterpret_cast<uint64_t*>(const_cast<int*>(s_flag) + 2);
@@ -590,12 +594,12 @@ __global__ void __launch_bounds__(kThreads, OCC) linear_ccw_kernel(const LinearP
   __syncthreads();
 
   if (warp == kConsumerWarps) {
-    produce<M, OCC == kCtasPerSmM1>(p, smem, full, empty, tag, w0, w1, lane);
+    produce<M, OCC != kCtasPerSm>(p, smem, full, empty, tag, w0, w1, lane);
     return;
   }
 
   pdl_wait();
-  if constexpr (OCC == kCtasPerSmM1) pdl_launch_dependents();
+  if constexpr (OCC != kCtasPerSm) pdl_launch_dependents();
   bool dead = false;
   if (PROBE && blockIdx.x == 0 && warp == 0) {
     // failure-path test: a bounded wait on a barrier that nothing completes and no copy
@@ -703,10 +707,11 @@ template <int M, int ES>
 sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, int kind, int occ, bool pdl) {
   void (*kern)(const LinearParams);
   if constexpr (M <= 4) {
-    if (occ == kCtasPerSmM1) {
+    if (occ == kCtasPerSmM1 || occ == kCtasPerSmM1b) {
       if constexpr (M == 1) {
         if (kind != 1 || p.cluster < 2 || p.probe_ns != 0) return SP_ERR_UNSUPPORTED;
-        kern = linear_ccw_kernel<1, ES, true, false, kCtasPerSmM1>;
+        kern = occ == kCtasPerSmM1 ? linear_ccw_kernel<1, ES, true, false, kCtasPerSmM1>
+                                   : linear_ccw_kernel<1, ES, true, false, kCtasPerSmM1b>;
       } else {
         return SP_ERR_UNSUPPORTED;
       }
@@ -722,13 +727,13 @@ sp_status launch_one(const LinearParams& p, cudaStream_t stream, size_t smem, in
   } else {
     kern = p.cluster > 1 ? linear_cc_kernel<M, ES, true> : linear_cc_kernel<M, ES, false>;
   }
-  static bool configured[4][2][kMaxDevices] = {};  // kernel attributes, once per device
+  static bool configured[5][2][kMaxDevices] = {};  // kernel attributes, once per device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= kMaxDevices) return SP_ERR_UNSUPPORTED;
   const int ci = p.cluster > 1 ? 1 : 0;
-  // the probe variant and the six-CTA variant are kernels of their own
-  const int ki = occ == kCtasPerSmM1 ? 3 : p.probe_ns != 0 ? 2 : kind;
+  // the probe variant and the six- and five-CTA variants are kernels of their own
+  const int ki = occ == kCtasPerSmM1 ? 3 : occ == kCtasPerSmM1b ? 4 : p.probe_ns != 0 ? 2 : kind;
   if (!configured[ki][ci][dev]) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemOptIn) != cudaSuccess ||
         (ci && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)) {
@@ -835,16 +840,19 @@ bool cc_plan(const sp_matrix* h, int Mt, int S, int occ, CcPlan* pl) {
   // tags (<= 64 B), the warps' partials (warp-per-chunk kernel) and the CTA's FP32
   // partial (cluster mode)
   const size_t part_bytes = S > 1 ? (size_t)kRows * Mt * sizeof(float) : 0;
-  const size_t comb_bytes = 2 * (size_t)kConsumerWarps * kRows * Mt * sizeof(float) + sizeof(FlushCtl);
+  // stream-K double-buffers the warps' partials (a warp may reach the next row block's end
+  // while the last one's is still being summed); a cluster CTA ends one row block
+  const size_t comb_bytes = (S > 1 ? 1 : 2) * (size_t)kConsumerWarps * kRows * Mt * sizeof(float) + sizeof(FlushCtl);
   pl->kind = 0;
   pl->occ = occ;
-  size_t ring = (occ == kCtasPerSmM1 ? kSmemBudgetM1 : kSmemBudget) - 256 - 16 - 64 - part_bytes;
+  size_t ring = (occ == kCtasPerSmM1 ? kSmemBudgetM1 : occ == kCtasPerSmM1b ? kSmemBudgetM1b : kSmemBudget) - 256 -
+                16 - 64 - part_bytes;
   if (Mt <= 4 && (ring - comb_bytes) / pl->slot_bytes >= (size_t)kConsumerWarps) {
     pl->kind = 1;
     ring -= comb_bytes;
   }
   pl->slots = (int)std::min<size_t>(16, ring / pl->slot_bytes);
-  if (pl->slots < 2 || (occ == kCtasPerSmM1 && pl->kind != 1)) return false;
+  if (pl->slots < 2 || (occ != kCtasPerSm && pl->kind != 1)) return false;
   pl->comb_off = (uint32_t)(((size_t)pl->slots * pl->slot_bytes + 2 * (size_t)pl->slots * 8 + 16 +
                              4 * (size_t)pl->slots + 15) /
                             16 * 16);
@@ -854,14 +862,16 @@ bool cc_plan(const sp_matrix* h, int Mt, int S, int occ, CcPlan* pl) {
 }
 
 // The launch configuration of one launch with Mt batch rows: six CTAs per SM for a
-// warp-per-chunk cluster launch at M = 1 where its plan fits, else four; S = 1 (stream-K)
-// without clusters.
+// warp-per-chunk cluster launch at M = 1 where its plan fits, else five where that fits,
+// else four; S = 1 (stream-K) without clusters.
 bool select_cc(const sp_matrix* h, int Mt, bool allow_cluster, bool probe, int* S, CcPlan* pl) {
   if (allow_cluster && Mt == 1 && !probe) {
-    const int s1 = cluster_cc(h, kCtasPerSmM1);
-    if (s1 > 1 && cc_plan(h, 1, s1, kCtasPerSmM1, pl)) {
-      *S = s1;
-      return true;
+    for (const int occ : {kCtasPerSmM1, kCtasPerSmM1b}) {
+      const int s1 = cluster_cc(h, occ);
+      if (s1 > 1 && cc_plan(h, 1, s1, occ, pl)) {
+        *S = s1;
+        return true;
+      }
     }
   }
   *S = allow_cluster ? cluster_cc(h, kCtasPerSm) : 1;
