@@ -10,6 +10,8 @@ from tests import test_oracle as pins
 
 SRC = os.path.join(os.path.dirname(oracle_mod.__file__), "sp_oracle.c")
 
+# Every mutant keeps the oracle's memory accesses inside its buffers (a mistake that
+# corrupts memory would end the test process rather than fail a pin).
 MUTANTS = {
     "sum_sign": ("acc += or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);",
                  "acc -= or_bf16_to_double(x[m * K + k]) * or_bf16_to_double(W[n * K + k]);"),
@@ -39,6 +41,19 @@ MUTANTS = {
     "update_grad_index": ("h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + k], w));",
                           "h = or_float_to_bf16_rne(fmaf(-lr, grad[n * K + (k ^ 1)], w));"),
     "bf16_shift": ("uint32_t u = (uint32_t)h << 16;", "uint32_t u = (uint32_t)h << 15;"),
+    "decompress_value_not_advanced": ("memcpy(Wb + (n * K + k) * esize, vals + v * esize, (size_t)esize);\n          ++v;",
+                                      "memcpy(Wb + (n * K + k) * esize, vals + v * esize, (size_t)esize);"),
+    "decompress_chunks_transposed": ("const uint8_t* chunk = buf + off[rb * T + t];\n      const uint8_t* vals = chunk + OR_MASK_BYTES;\n      int64_t v = 0;\n      for (int r = 0; r < OR_CHUNK_ROWS; ++r) {\n        int64_t n = rb * OR_CHUNK_ROWS + r;\n        uint64_t m = or_read_u64le",
+                                     "const uint8_t* chunk = buf + off[t * RB + rb];\n      const uint8_t* vals = chunk + OR_MASK_BYTES;\n      int64_t v = 0;\n      for (int r = 0; r < OR_CHUNK_ROWS; ++r) {\n        int64_t n = rb * OR_CHUNK_ROWS + r;\n        uint64_t m = or_read_u64le"),
+    "from_format_byte_swap": ("uint16_t h = (uint16_t)(vals[2 * v] | (vals[2 * v + 1] << 8));",
+                              "uint16_t h = (uint16_t)(vals[2 * v + 1] | (vals[2 * v] << 8));"),
+    "from_format_neighbour_mask": ("uint64_t msk = or_read_u64le(chunk + r * 8);",
+                                   "uint64_t msk = or_read_u64le(chunk + (r ^ 1) * 8);"),
+    "from_format_int8_unscaled": ("w = (double)(int8_t)vals[v] * (double)scale[n];", "w = (double)(int8_t)vals[v];"),
+    "from_format_int8_unsigned": ("w = (double)(int8_t)vals[v] * (double)scale[n];",
+                                  "w = (double)vals[v] * (double)scale[n];"),
+    "residual_h_dropped": ("out[m * N + j] = or_bf16_to_double(h[m * N + j]) + or_bf16_to_double(a[m * N + j])",
+                           "out[m * N + j] = or_bf16_to_double(a[m * N + j]) + or_bf16_to_double(a[m * N + j])"),
     "tile_width_off_by_one": ("for (int j = 0; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals",
                               "for (int j = 1; j < OR_TILE_K; ++j) {\n          if (!((m >> j) & 1u)) continue;\n          int64_t k = t * OR_TILE_K + j;\n          memcpy(vals"),
 }
@@ -57,6 +72,7 @@ def _pin_suite(o):
         "integer_exact": lambda: pins.test_linear_integer_valued_exact(o, 40, 136, 3),
         "library_matmul": lambda: pins.test_linear_matches_float64_library_matmul(o, 70),
         "one_hot": lambda: pins.test_linear_one_hot_selects_a_column(o),
+        "from_format_def": lambda: pins.test_linear_from_format_bitwise_equals_definition(o),
         "int8_exact": lambda: pins.test_int8_oracle_integer_exact_and_scale(o),
         "glue": lambda: pins.test_glue_hand_derived_values(o),
         "w8a8_int": lambda: pins.test_w8a8_integer_sum_equals_int64_matmul(o),
