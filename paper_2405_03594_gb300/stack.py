@@ -1,15 +1,19 @@
 """Decode step of a Llama-2-7B linear-only stack on libsp.
 
-Per layer, four fused sparse linears and the elementwise glue of include/sp_stack.h:
+Per layer, four sparse linears and the elementwise glue of include/sp_stack.h:
 
     qkv = x.Wqkv^T            [M, 12288]      (sparse linear)
-    v   = qkv[:, 8192:12288]                   (sp_copy_columns)
-    h   = h + v.Wo^T + r_l                      (sparse linear, sp_residual_add)
-    gu  = h.Wgu^T             [M, 22016]      (sparse linear)
-    a   = gu[:, :11008] * gu[:, 11008:]        (sp_mul_halves)
-    h   = h + a.Wdown^T + r'_l                  (sparse linear, sp_residual_add)
+    v   = qkv[:, 8192:12288]                   (read in place at M = 1, else sp_copy_columns)
+    h   = h + v.Wo^T + r_l                      (sparse linear + residual)
+    a   = gate(h) * up(h)     [M, 11008]      (sparse linear + gate * up)
+    h   = h + a.Wdown^T + r'_l                  (sparse linear + residual)
 
-All arithmetic runs in libsp kernels; PyTorch only holds the buffers.  The layers are
+By default (`fused`) the gate/up weight holds interleaved rows (gate_j, up_j), and where a
+batch runs on the CUDA-core decode kernels the residual adds and the gate * up product are
+those kernels' output epilogues (sp_linear_epi): four launches per layer.  Tensor-core
+batches, and stacks built with fused=False, run each linear into a buffer and the glue as
+its own launch (sp_residual_add; sp_mul_pairs on interleaved rows, sp_mul_halves on the
+[gate, up] layout).  All arithmetic runs in libsp kernels; PyTorch only holds the buffers.  The layers are
 device copies of one seeded layer (each its own HBM buffers, so a step streams the full
 32-layer weight set), or each layer's own seeded inputs (`host_layers`: distinct weights,
 or a per-layer sparsity profile).  `capture()` records one step as a single CUDA graph.
